@@ -1,0 +1,305 @@
+/*
+ * mk_oracle.c -- plain fp64 CPU oracle for the attention forward pass.
+ *
+ * TEST INFRASTRUCTURE.  Only tests/, __graft_entry__.smoke() and bench.py's
+ * cpu_baseline / reference legs may load this file's library.  The product
+ * path (the CUDA library and its Python binding) never calls it and shares
+ * no code with it.
+ *
+ * What it computes.  The paper's problem statement (Section 2.1, the Testing
+ * and Verification Agents; Section 3.1, correctness against the unoptimized
+ * reference implementation) fixes the contract: a kernel takes the same input
+ * arrays as the reference operation and must return the same outputs.  The
+ * reference operation for the Flash Attention and GQA Attention rows of
+ * Table 2 is the plain definition of scaled dot-product attention, which this
+ * file writes out directly, with no tiling, no online softmax and no
+ * reordering:
+ *
+ *   for each sequence b, query head h (key/value head g = h / (Hq / Hkv)),
+ *   and query position i of that sequence:
+ *     K_i  = { j : 0 <= j < L_b  and  (not causal  or  j <= i) }
+ *     s_j  = scale * sum_d q[b,i,h,d] * k[b,j,g,d]          (j in K_i)
+ *     m    = max_j s_j
+ *     l    = sum_j exp(s_j - m)
+ *     o[d] = sum_j exp(s_j - m) * v[b,j,g,d] / l
+ *     lse  = m + ln(l)                                        (natural log)
+ *
+ * Subtracting m is the textbook overflow guard; it cancels exactly in o and
+ * is added back in lse, so the result is the definition itself.
+ *
+ * Inputs are bf16 bit patterns (uint16); they are widened exactly to fp64.
+ * All arithmetic is fp64.  Layouts:
+ *   fixed length (cu_seqlens == NULL): q/o [B,S,Hq,D], k/v [B,S,Hkv,D],
+ *                                      lse [B,Hq,S]
+ *   packed varlen (cu_seqlens != NULL): q/o [T,Hq,D], k/v [T,Hkv,D],
+ *                                      lse [Hq,T], T = S = cu_seqlens[B]
+ * Readings where the paper is silent: contiguous query-head groups
+ * (g = h / (Hq/Hkv)); causal alignment with Sq == Sk, so row i sees keys
+ * 0..i; the log-sum-exp includes the scale and uses the natural log.
+ * A row with no visible key (cannot happen for valid inputs) gets o = 0,
+ * lse = -inf.
+ */
+#include <math.h>
+#include <pthread.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define MK_ORACLE_OK 0
+#define MK_ORACLE_BAD_ARG (-1)
+#define MK_ORACLE_NO_MEM (-2)
+
+static double bf16_bits_to_f64(uint16_t bits)
+{
+    uint32_t u = ((uint32_t)bits) << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+typedef struct {
+    const uint16_t *q, *k, *v;
+    int B, Hq, Hkv, S, D, causal;
+    double scale;
+    const int32_t *cu;
+} problem_t;
+
+/* Token offset and length of sequence b. */
+static void seq_bounds(const problem_t *p, int b, int64_t *tok0, int *len)
+{
+    if (p->cu) {
+        *tok0 = p->cu[b];
+        *len = p->cu[b + 1] - p->cu[b];
+    } else {
+        *tok0 = (int64_t)b * p->S;
+        *len = p->S;
+    }
+}
+
+/* One output row: the definition above for (sequence b, head h, position i).
+ * s_buf must hold at least L_b doubles. */
+static void attention_row(const problem_t *p, int b, int h, int i, double *s_buf,
+                          double *o_row, double *lse_out)
+{
+    const int D = p->D;
+    const int group = p->Hq / p->Hkv;
+    const int g = h / group;
+    int64_t tok0;
+    int L;
+    seq_bounds(p, b, &tok0, &L);
+
+    const uint16_t *qi = p->q + ((tok0 + i) * p->Hq + h) * (int64_t)D;
+    int n_keys = p->causal ? (i + 1 < L ? i + 1 : L) : L; /* |K_i| */
+
+    double m = -INFINITY;
+    for (int j = 0; j < n_keys; ++j) {
+        const uint16_t *kj = p->k + ((tok0 + j) * p->Hkv + g) * (int64_t)D;
+        double dot = 0.0;
+        for (int d = 0; d < D; ++d)
+            dot += bf16_bits_to_f64(qi[d]) * bf16_bits_to_f64(kj[d]);
+        double s = p->scale * dot;
+        s_buf[j] = s;
+        if (s > m)
+            m = s;
+    }
+
+    for (int d = 0; d < D; ++d)
+        o_row[d] = 0.0;
+    if (n_keys == 0) {
+        *lse_out = -INFINITY;
+        return;
+    }
+
+    double l = 0.0;
+    for (int j = 0; j < n_keys; ++j) {
+        const uint16_t *vj = p->v + ((tok0 + j) * p->Hkv + g) * (int64_t)D;
+        double w = exp(s_buf[j] - m);
+        l += w;
+        for (int d = 0; d < D; ++d)
+            o_row[d] += w * bf16_bits_to_f64(vj[d]);
+    }
+    for (int d = 0; d < D; ++d)
+        o_row[d] /= l;
+    *lse_out = m + log(l);
+}
+
+static int check_problem(const problem_t *p)
+{
+    if (!p->q || !p->k || !p->v)
+        return MK_ORACLE_BAD_ARG;
+    if (p->B < 1 || p->Hq < 1 || p->Hkv < 1 || p->S < 0 || p->D < 1)
+        return MK_ORACLE_BAD_ARG;
+    if (p->Hq % p->Hkv != 0)
+        return MK_ORACLE_BAD_ARG;
+    if (p->cu) {
+        if (p->cu[0] != 0 || p->cu[p->B] != p->S)
+            return MK_ORACLE_BAD_ARG;
+        for (int b = 0; b < p->B; ++b)
+            if (p->cu[b + 1] < p->cu[b])
+                return MK_ORACLE_BAD_ARG;
+    }
+    return MK_ORACLE_OK;
+}
+
+static int max_seq_len(const problem_t *p)
+{
+    int mx = 0;
+    for (int b = 0; b < p->B; ++b) {
+        int64_t t0;
+        int L;
+        seq_bounds(p, b, &t0, &L);
+        if (L > mx)
+            mx = L;
+    }
+    return mx;
+}
+
+/* ---------------------------------------------------------------- full pass */
+
+typedef struct {
+    const problem_t *p;
+    double *o, *lse;
+    int64_t n_tasks;   /* (b, h) pairs */
+    int64_t *next;     /* shared task counter */
+    int max_len;
+    int status;
+} full_job_t;
+
+static void *full_worker(void *arg)
+{
+    full_job_t *job = (full_job_t *)arg;
+    const problem_t *p = job->p;
+    double *s_buf = (double *)malloc(sizeof(double) * (size_t)(job->max_len > 0 ? job->max_len : 1));
+    if (!s_buf) {
+        job->status = MK_ORACLE_NO_MEM;
+        return NULL;
+    }
+    for (;;) {
+        int64_t t = __atomic_fetch_add(job->next, 1, __ATOMIC_RELAXED);
+        if (t >= job->n_tasks)
+            break;
+        int b = (int)(t / p->Hq), h = (int)(t % p->Hq);
+        int64_t tok0;
+        int L;
+        seq_bounds(p, b, &tok0, &L);
+        for (int i = 0; i < L; ++i) {
+            double *o_row = job->o + ((tok0 + i) * p->Hq + h) * (int64_t)p->D;
+            int64_t lse_idx = p->cu ? (int64_t)h * p->S + tok0 + i
+                                    : ((int64_t)b * p->Hq + h) * p->S + i;
+            attention_row(p, b, h, i, s_buf, o_row, &job->lse[lse_idx]);
+        }
+    }
+    free(s_buf);
+    return NULL;
+}
+
+/* Runs `worker` on n_threads threads, each given its own copy of *job
+ * (the copies share the task counter). */
+static int run_threads(void *(*worker)(void *), void *job, size_t job_size, int n_threads)
+{
+    if (n_threads < 1)
+        n_threads = 1;
+    pthread_t *tids = (pthread_t *)calloc((size_t)n_threads, sizeof(pthread_t));
+    char *jobs = (char *)malloc(job_size * (size_t)n_threads);
+    if (!tids || !jobs) {
+        free(tids);
+        free(jobs);
+        return MK_ORACLE_NO_MEM;
+    }
+    int started = 0;
+    for (int t = 0; t < n_threads; ++t) {
+        memcpy(jobs + job_size * t, job, job_size);
+        if (pthread_create(&tids[t], NULL, worker, jobs + job_size * t) != 0)
+            break;
+        ++started;
+    }
+    if (started == 0) /* no thread could start: do the work here */
+        worker(jobs);
+    for (int t = 0; t < started; ++t)
+        pthread_join(tids[t], NULL);
+    free(tids);
+    free(jobs);
+    return MK_ORACLE_OK;
+}
+
+/*
+ * Full forward pass.  o has the layout of q; lse as described above.
+ * Returns 0, or a negative code for invalid arguments / allocation failure.
+ */
+int mk_oracle_attn_fwd_f64(const uint16_t *q, const uint16_t *k, const uint16_t *v,
+                           double *o, double *lse, int B, int Hq, int Hkv, int S, int D,
+                           int causal, double scale, const int32_t *cu_seqlens,
+                           int n_threads)
+{
+    problem_t p = {q, k, v, B, Hq, Hkv, S, D, causal != 0, scale, cu_seqlens};
+    int st = check_problem(&p);
+    if (st != MK_ORACLE_OK)
+        return st;
+    if (!o || !lse)
+        return MK_ORACLE_BAD_ARG;
+    int64_t next = 0;
+    full_job_t job = {&p, o, lse, (int64_t)B * Hq, &next, max_seq_len(&p), MK_ORACLE_OK};
+    st = run_threads(full_worker, &job, sizeof job, n_threads);
+    return st;
+}
+
+/* ------------------------------------------------------------ sampled rows */
+
+typedef struct {
+    const problem_t *p;
+    const int64_t *rows; /* n_rows x 3: (b, h, i) */
+    double *o_rows;      /* n_rows x D */
+    double *lse_rows;    /* n_rows */
+    int64_t n_rows;
+    int64_t *next;
+    int max_len;
+} rows_job_t;
+
+static void *rows_worker(void *arg)
+{
+    rows_job_t *job = (rows_job_t *)arg;
+    const problem_t *p = job->p;
+    double *s_buf = (double *)malloc(sizeof(double) * (size_t)(job->max_len > 0 ? job->max_len : 1));
+    if (!s_buf)
+        return NULL;
+    for (;;) {
+        int64_t r = __atomic_fetch_add(job->next, 1, __ATOMIC_RELAXED);
+        if (r >= job->n_rows)
+            break;
+        int b = (int)job->rows[3 * r], h = (int)job->rows[3 * r + 1], i = (int)job->rows[3 * r + 2];
+        attention_row(p, b, h, i, s_buf, job->o_rows + r * (int64_t)p->D, &job->lse_rows[r]);
+    }
+    free(s_buf);
+    return NULL;
+}
+
+/*
+ * The same definition evaluated only on selected rows (b, h, i), for inputs
+ * too large to evaluate in full.  Each row is independent of the others, so a
+ * sampled row equals the corresponding row of mk_oracle_attn_fwd_f64.
+ */
+int mk_oracle_attn_rows_f64(const uint16_t *q, const uint16_t *k, const uint16_t *v,
+                            int B, int Hq, int Hkv, int S, int D, int causal, double scale,
+                            const int32_t *cu_seqlens, const int64_t *rows, int64_t n_rows,
+                            double *o_rows, double *lse_rows, int n_threads)
+{
+    problem_t p = {q, k, v, B, Hq, Hkv, S, D, causal != 0, scale, cu_seqlens};
+    int st = check_problem(&p);
+    if (st != MK_ORACLE_OK)
+        return st;
+    if (n_rows < 0 || (n_rows > 0 && (!rows || !o_rows || !lse_rows)))
+        return MK_ORACLE_BAD_ARG;
+    for (int64_t r = 0; r < n_rows; ++r) {
+        int b = (int)rows[3 * r], h = (int)rows[3 * r + 1], i = (int)rows[3 * r + 2];
+        if (b < 0 || b >= B || h < 0 || h >= Hq || i < 0)
+            return MK_ORACLE_BAD_ARG;
+        int64_t t0;
+        int L;
+        seq_bounds(&p, b, &t0, &L);
+        if (i >= L)
+            return MK_ORACLE_BAD_ARG;
+    }
+    int64_t next = 0;
+    rows_job_t job = {&p, rows, o_rows, lse_rows, n_rows, &next, max_seq_len(&p)};
+    return run_threads(rows_worker, &job, sizeof job, n_threads);
+}

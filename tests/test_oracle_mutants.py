@@ -1,0 +1,59 @@
+"""Planted mistakes in the oracle fail its pins (no GPU).
+
+Each mutant is a copy of oracle/mk_oracle.c with one plausible mistake (a
+dropped term, a wrong sign or index, a swapped operand, an off-by-one mask,
+the wrong logarithm, a wrong output index), compiled to a temporary library.
+The pin suite in oracle_pin_checks.py must reject every one of them; the real
+oracle passes it (test_oracle_pins.py)."""
+import os
+
+import pytest
+
+import oracle
+import oracle_pin_checks as pins
+
+SRC = os.path.join(os.path.dirname(oracle.__file__), "mk_oracle.c")
+
+MUTANTS = {
+    "drop_scale": ("double s = p->scale * dot;", "double s = dot;"),
+    "sign_of_max": ("double w = exp(s_buf[j] - m);", "double w = exp(s_buf[j] + m);"),
+    "lse_without_max": ("*lse_out = m + log(l);", "*lse_out = log(l);"),
+    "lse_log2": ("*lse_out = m + log(l);", "*lse_out = m + log2(l);"),
+    "no_normalisation": ("        o_row[d] /= l;\n    *lse_out", "        o_row[d] *= 1.0;\n    *lse_out"),
+    "causal_excludes_diagonal": ("int n_keys = p->causal ? (i + 1 < L ? i + 1 : L) : L;",
+                                 "int n_keys = p->causal ? (i < L ? i : L) : L;"),
+    "causal_ignored": ("int n_keys = p->causal ? (i + 1 < L ? i + 1 : L) : L;",
+                       "int n_keys = L;"),
+    "gqa_interleaved_groups": ("const int g = h / group;", "const int g = h % p->Hkv;"),
+    "keys_read_from_values": ("const uint16_t *kj = p->k + ", "const uint16_t *kj = p->v + "),
+    "values_read_from_keys": ("const uint16_t *vj = p->v + ", "const uint16_t *vj = p->k + "),
+    "query_row_offset": ("const uint16_t *qi = p->q + ((tok0 + i) * p->Hq + h)",
+                         "const uint16_t *qi = p->q + ((tok0 + i) * p->Hq + 0)"),
+    "varlen_lse_index": ("int64_t lse_idx = p->cu ? (int64_t)h * p->S + tok0 + i",
+                         "int64_t lse_idx = p->cu ? (int64_t)h * p->S + i"),
+    "weights_not_accumulated": ("        l += w;\n", "        l = w;\n"),
+    "last_dim_dropped": ("for (int d = 0; d < D; ++d)\n            dot +=",
+                         "for (int d = 0; d + 1 < D; ++d)\n            dot +="),
+}
+
+
+@pytest.fixture(scope="module")
+def source():
+    with open(SRC) as f:
+        return f.read()
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_mutant_is_caught(tmp_path, source, name):
+    old, new = MUTANTS[name]
+    assert source.count(old) == 1, f"mutation site for {name} not found exactly once"
+    src = tmp_path / f"mutant_{name}.c"
+    src.write_text(source.replace(old, new))
+    lib = oracle.load(oracle.compile_oracle(str(src), str(tmp_path / f"libmutant_{name}.so")))
+    failures = []
+    for check in pins.ALL_CHECKS:
+        try:
+            check(lib)
+        except AssertionError as e:
+            failures.append(f"{check.__name__}: {e}")
+    assert failures, f"mutant {name} passed every pin"
