@@ -1,0 +1,104 @@
+/*
+ * mk_attn.h -- C ABI of the GB300 (sm_103a) attention forward library.
+ *
+ * The operation is the fused attention forward pass whose reference the
+ * paper's Flash Attention and GQA Attention kernels reproduce (Table 2; the
+ * contract of Section 2.1 and Section 3.1: take the same input arrays as the
+ * reference operation and return the same outputs).  For each sequence b,
+ * query head h (key/value head g = h / (Hq / Hkv), contiguous groups) and
+ * query position i of the sequence:
+ *
+ *   K_i    = { j : 0 <= j < L_b  and  (not causal  or  j <= i) }
+ *   o[i]   = sum_{j in K_i} softmax_j(scale * q[i] . k[j]) * v[j]
+ *   lse[i] = ln( sum_{j in K_i} exp(scale * q[i] . k[j]) )        (natural log)
+ *
+ * Causal masking is aligned top-left: query and key sequences have the same
+ * length, so row i sees keys 0..i.
+ *
+ * Everything here is plain C: device pointers, sizes and a CUDA stream handle
+ * passed as void*.  No symbol takes a PyTorch type.
+ */
+#ifndef MK_ATTN_H
+#define MK_ATTN_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define MK_API __attribute__((visibility("default")))
+#else
+#define MK_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status codes returned by every entry point. */
+typedef enum {
+    MK_OK = 0,
+    MK_ERR_INVALID_ARG = -1,  /* null pointer, non-positive size, Hq % Hkv != 0 */
+    MK_ERR_UNSUPPORTED = -2,  /* head dimension other than 64 or 128 */
+    MK_ERR_ALIGNMENT = -3,    /* a base pointer not 16-byte aligned */
+    MK_ERR_CUDA = -4,         /* a CUDA runtime/driver call failed */
+    MK_ERR_TIMEOUT = -5       /* a kernel wait ran out; reported by mk_attn_check_status */
+} mk_status;
+
+/*
+ * mk_attn_fwd -- attention forward pass (causal or not, GQA, optional varlen).
+ *
+ * Arguments (all pointers are DEVICE pointers owned by the caller):
+ *   q          bf16, fixed length [B, S, Hq, D]; varlen [T, Hq, D]. Read only.
+ *   k, v       bf16, fixed length [B, S, Hkv, D]; varlen [T, Hkv, D]. Read only.
+ *   o          bf16 output, same layout as q.  Fully overwritten.
+ *   lse        fp32 output, fixed length [B, Hq, S]; varlen [Hq, T].  Fully
+ *              overwritten with the natural-log row log-sum-exp (scale included).
+ *   B          number of sequences (>= 1).
+ *   Hq, Hkv    query and key/value heads (>= 1, Hq % Hkv == 0).
+ *   S          fixed length: tokens per sequence (>= 1);
+ *              varlen: total tokens T = cu_seqlens[B] (>= 1).
+ *   D          head dimension, 64 or 128.
+ *   causal     nonzero: row i attends to keys 0..i of its sequence.
+ *   scale      multiplier of q . k before the softmax (e.g. 1/sqrt(D)).
+ *   cu_seqlens NULL for fixed length; otherwise a DEVICE int32 array [B+1]
+ *              of sequence start offsets into the packed token dimension:
+ *              cu_seqlens[0] = 0, non-decreasing, cu_seqlens[B] = T.  It is
+ *              read only on the device, so the call never synchronises.
+ *              Values outside [0, T] are clamped on the device: a malformed
+ *              array gives unspecified results but no access outside q, k, v,
+ *              o and lse.
+ *   stream     cudaStream_t (NULL = legacy default stream).
+ *
+ * Layout: every tensor is contiguous, innermost dimension last; each base
+ * pointer must be 16-byte aligned.
+ *
+ * Behaviour: the call validates its arguments on the host, encodes TMA
+ * descriptors and enqueues one kernel on `stream`; it returns without
+ * synchronising.  On any error it returns a negative mk_status and enqueues
+ * nothing, so o and lse are left untouched.  The library allocates no device
+ * memory.  Results are deterministic: no atomics, so repeated calls on the same
+ * inputs are bitwise identical.  Sequences of length 0 (varlen) produce no
+ * rows.  Every internal wait of the kernel is bounded; if one runs out the
+ * kernel records MK_ERR_TIMEOUT for mk_attn_check_status and exits.
+ */
+MK_API int mk_attn_fwd(const void *q, const void *k, const void *v, void *o, float *lse,
+                       int B, int Hq, int Hkv, int S, int D, int causal, float scale,
+                       const int32_t *cu_seqlens, void *stream);
+
+/* Short static description of a status code.  Never NULL. */
+MK_API const char *mk_attn_error_string(int status);
+
+/*
+ * mk_attn_check_status -- synchronises `stream`, then reads and clears the
+ * device status word written by kernels whose internal waits ran out.
+ * Returns MK_OK, MK_ERR_TIMEOUT, or MK_ERR_CUDA if synchronisation failed.
+ */
+MK_API int mk_attn_check_status(void *stream);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+MK_API int mk_attn_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MK_ATTN_H */

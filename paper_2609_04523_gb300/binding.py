@@ -1,0 +1,135 @@
+"""Thin ctypes binding of the C ABI in include/mk_attn.h.
+
+Argument marshalling only: every step of the attention forward pass runs in
+the CUDA library.  There is no CPU or PyTorch fallback; if the library is
+missing or cannot be loaded, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG, "libmk_attn.so")
+
+MK_OK = 0
+MK_ERR_INVALID_ARG = -1
+MK_ERR_UNSUPPORTED = -2
+MK_ERR_ALIGNMENT = -3
+MK_ERR_CUDA = -4
+MK_ERR_TIMEOUT = -5
+
+# Symbols declared in include/mk_attn.h.
+EXPORTED = ("mk_attn_fwd", "mk_attn_error_string", "mk_attn_check_status", "mk_attn_version")
+
+_lock = threading.Lock()
+_lib = None
+
+
+class MkAttnError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"{msg} (status {status})")
+        self.status = status
+
+
+def library_path() -> str:
+    return LIB_PATH
+
+
+def load_library() -> ctypes.CDLL:
+    """Loads the in-tree CUDA library; raises if it has not been built."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB_PATH):
+                raise MkAttnError(MK_ERR_CUDA,
+                                  f"CUDA library not built: {LIB_PATH} is missing "
+                                  "(run paper_2609_04523_gb300.build.build_library())")
+            lib = ctypes.CDLL(LIB_PATH)
+            vp, i = ctypes.c_void_p, ctypes.c_int
+            lib.mk_attn_fwd.argtypes = [vp, vp, vp, vp, vp, i, i, i, i, i, i, ctypes.c_float,
+                                        vp, vp]
+            lib.mk_attn_fwd.restype = i
+            lib.mk_attn_error_string.argtypes = [i]
+            lib.mk_attn_error_string.restype = ctypes.c_char_p
+            lib.mk_attn_check_status.argtypes = [vp]
+            lib.mk_attn_check_status.restype = i
+            lib.mk_attn_version.argtypes = []
+            lib.mk_attn_version.restype = i
+            _lib = lib
+    return _lib
+
+
+def mk_attn_fwd(q: int, k: int, v: int, o: int, lse: int, B: int, Hq: int, Hkv: int, S: int,
+                D: int, causal: int, scale: float, cu_seqlens: int | None, stream: int | None) -> int:
+    """Raw C-ABI call: integer device pointers in, status code out."""
+    return load_library().mk_attn_fwd(q, k, v, o, lse, B, Hq, Hkv, S, D, int(causal),
+                                      float(scale), cu_seqlens, stream)
+
+
+def mk_attn_error_string(status: int) -> str:
+    return load_library().mk_attn_error_string(int(status)).decode()
+
+
+def mk_attn_check_status(stream: int | None) -> int:
+    return load_library().mk_attn_check_status(stream)
+
+
+def mk_attn_version() -> int:
+    return load_library().mk_attn_version()
+
+
+def _check(status: int):
+    if status != MK_OK:
+        raise MkAttnError(status, mk_attn_error_string(status))
+
+
+def attn_fwd(q, k, v, causal: bool = True, scale: float | None = None, cu_seqlens=None,
+             out=None, lse=None, stream=None):
+    """Attention forward on CUDA tensors through mk_attn_fwd.
+
+    q: [B,S,Hq,D] bf16 (or [T,Hq,D] with cu_seqlens, an int32 CUDA tensor
+    [B+1]); k, v: [B,S,Hkv,D] (or [T,Hkv,D]).  Returns (o, lse): o like q (bf16),
+    lse fp32 [B,Hq,S] (or [Hq,T]).  PyTorch only allocates the outputs and
+    provides the stream."""
+    import torch
+    if not (q.is_cuda and k.is_cuda and v.is_cuda):
+        raise ValueError("q, k, v must be CUDA tensors")
+    if q.dtype != torch.bfloat16 or k.dtype != torch.bfloat16 or v.dtype != torch.bfloat16:
+        raise ValueError("q, k, v must be bfloat16")
+    if not (q.is_contiguous() and k.is_contiguous() and v.is_contiguous()):
+        raise ValueError("q, k, v must be contiguous")
+    if cu_seqlens is None:
+        if q.dim() != 4 or k.dim() != 4 or k.shape != v.shape:
+            raise ValueError("fixed-length layout is q [B,S,Hq,D], k/v [B,S,Hkv,D]")
+        B, S, Hq, D = q.shape
+        Hkv = k.shape[2]
+        if k.shape[0] != B or k.shape[1] != S or k.shape[3] != D:
+            raise ValueError("k/v shape does not match q")
+        lse_shape = (B, Hq, S)
+        cu_ptr = None
+    else:
+        if q.dim() != 3 or k.dim() != 3 or k.shape != v.shape:
+            raise ValueError("varlen layout is q [T,Hq,D], k/v [T,Hkv,D]")
+        if not cu_seqlens.is_cuda or cu_seqlens.dtype != torch.int32 or cu_seqlens.dim() != 1:
+            raise ValueError("cu_seqlens must be a 1-D int32 CUDA tensor")
+        S, Hq, D = q.shape
+        Hkv = k.shape[1]
+        B = cu_seqlens.numel() - 1
+        if k.shape[0] != S or k.shape[2] != D:
+            raise ValueError("k/v shape does not match q")
+        lse_shape = (Hq, S)
+        cu_ptr = cu_seqlens.data_ptr()
+    if scale is None:
+        scale = 1.0 / float(D) ** 0.5
+    if out is None:
+        out = torch.empty_like(q)
+    if lse is None:
+        lse = torch.empty(lse_shape, dtype=torch.float32, device=q.device)
+    if stream is None:
+        stream = torch.cuda.current_stream(q.device)
+    _check(mk_attn_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), lse.data_ptr(),
+                       B, Hq, Hkv, S, D, int(bool(causal)), float(scale), cu_ptr,
+                       stream.cuda_stream))
+    return out, lse

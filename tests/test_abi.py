@@ -1,0 +1,88 @@
+"""The C-ABI library loads, exports what include/*.h declares, and rejects
+invalid arguments on the host before any CUDA call (no GPU needed)."""
+import glob
+import os
+import re
+
+import pytest
+
+from paper_2609_04523_gb300 import binding
+from paper_2609_04523_gb300.build import build_library
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build_library()
+    return binding.load_library()
+
+
+def declared_symbols():
+    names = set()
+    for h in glob.glob(os.path.join(ROOT, "include", "*.h")):
+        text = open(h).read()
+        names |= set(re.findall(r"MK_API\s+[\w\s\*]*?\b(mk_\w+)\s*\(", text))
+    return names
+
+
+def test_header_declares_the_entry_points():
+    assert {"mk_attn_fwd", "mk_attn_error_string", "mk_attn_check_status",
+            "mk_attn_version"} <= declared_symbols()
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in declared_symbols():
+        assert hasattr(lib, name), f"{name} declared in include/ but not exported"
+
+
+def test_version_and_error_strings(lib):
+    assert binding.mk_attn_version() >= 100
+    for st in (0, -1, -2, -3, -4, -5, -99):
+        assert isinstance(binding.mk_attn_error_string(st), str)
+    assert "align" in binding.mk_attn_error_string(binding.MK_ERR_ALIGNMENT)
+
+
+A = 0x10000  # fake 16-byte-aligned addresses: never dereferenced by a rejected call
+GOOD = dict(q=A, k=2 * A, v=3 * A, o=4 * A, lse=5 * A, B=2, Hq=8, Hkv=2, S=256, D=128,
+            causal=1, scale=0.088, cu_seqlens=None, stream=None)
+
+
+def call(**kw):
+    args = dict(GOOD)
+    args.update(kw)
+    return binding.mk_attn_fwd(**args)
+
+
+@pytest.mark.parametrize("kw, want", [
+    (dict(q=None), binding.MK_ERR_INVALID_ARG),
+    (dict(k=None), binding.MK_ERR_INVALID_ARG),
+    (dict(v=None), binding.MK_ERR_INVALID_ARG),
+    (dict(o=None), binding.MK_ERR_INVALID_ARG),
+    (dict(lse=None), binding.MK_ERR_INVALID_ARG),
+    (dict(B=0), binding.MK_ERR_INVALID_ARG),
+    (dict(S=0), binding.MK_ERR_INVALID_ARG),
+    (dict(Hq=0), binding.MK_ERR_INVALID_ARG),
+    (dict(Hkv=0), binding.MK_ERR_INVALID_ARG),
+    (dict(Hkv=3), binding.MK_ERR_INVALID_ARG),
+    (dict(B=-1), binding.MK_ERR_INVALID_ARG),
+    (dict(scale=float("nan")), binding.MK_ERR_INVALID_ARG),
+    (dict(scale=float("inf")), binding.MK_ERR_INVALID_ARG),
+    (dict(D=96), binding.MK_ERR_UNSUPPORTED),
+    (dict(D=256), binding.MK_ERR_UNSUPPORTED),
+    (dict(D=0), binding.MK_ERR_UNSUPPORTED),
+    (dict(q=A + 8), binding.MK_ERR_ALIGNMENT),
+    (dict(o=A + 2), binding.MK_ERR_ALIGNMENT),
+    (dict(lse=A + 4), binding.MK_ERR_ALIGNMENT),
+    (dict(cu_seqlens=A + 2), binding.MK_ERR_ALIGNMENT),
+    (dict(B=1 << 20, S=1 << 12), binding.MK_ERR_INVALID_ARG),  # token count overflows int32
+])
+def test_invalid_arguments_rejected_on_host(lib, kw, want):
+    assert call(**kw) == want
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    monkeypatch.setattr(binding, "_lib", None)
+    monkeypatch.setattr(binding, "LIB_PATH", str(tmp_path / "absent.so"))
+    with pytest.raises(binding.MkAttnError):
+        binding.load_library()
