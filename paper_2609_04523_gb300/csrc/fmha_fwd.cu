@@ -6,23 +6,32 @@
 // and GQA Attention kernels (Table 2), under the contract of Section 2.1 and
 // Section 3.1 (same inputs and outputs as the reference operation).
 //
-// Design (one CTA = one 128-row query tile of one (sequence, query head)):
-//   warp 5 (one thread)  TMA producer: the Q tile once, then K_j and V_j blocks of
-//                        128 keys through an n-stage shared-memory ring
-//                        (128-byte swizzle, mbarrier transaction counts).
-//   warp 4 (one thread)  tcgen05 MMA issuer: S_j = Q K_j^T into one of two TMEM
-//                        S buffers (fp32), and O += P_j V_j with P_j read from
-//                        TMEM (bf16, written over S_j) and V_j as an MN-major
-//                        shared-memory operand.
-//   warps 0-3            softmax: thread r owns query row r, i.e. TMEM lane r.
-//                        Online softmax in base 2 (t = s * scale * log2 e),
-//                        lazy O rescaling (only when the row max rises by more
-//                        than kRescaleThreshold), P rounded to bf16 (RNE) into
-//                        TMEM; then the epilogue O / l -> bf16 and
-//                        lse = ln 2 * (m + log2 l).
-// Causal tiles visit key blocks 0..qt only (block skipping) and mask only the
-// diagonal block; the ragged tail of a sequence is masked by key position.
-// TMEM: S0 = columns 0..127, S1 = 128..255, O = 256..256+D.
+// Design: persistent CTAs, one per SM.  A work unit is a pair of 128-row query
+// tiles (A = rows 256p..256p+127, B = the next 128) of one (sequence, query
+// head); both tiles share every K/V block the producer loads.  Roles:
+//   warps 0-3   softmax of tile A, thread r owns row r = TMEM lane r
+//   warps 4-7   softmax of tile B (same lanes, warp % 4 selects the lane quarter)
+//   warp 8      tcgen05 MMA issuer (one thread)
+//   warp 9      TMA producer (one thread): Q_A, Q_B per unit, then K_j, V_j
+//               blocks of 128 keys through an n-stage 128-byte-swizzled ring
+//   warps 10-11 idle (they complete the third warpgroup)
+// Registers: the block launches with 168 per thread (384 threads); the third
+// warpgroup gives back down to kRegsCtl and the two softmax warpgroups grow to
+// kRegsSoftmax, so each SM sub-partition (one warp of each warpgroup) stays
+// within its 16K registers: 2 * 208 + 80 = 496 <= 3 * 168.
+// TMEM (512 columns): S_A = 0..127, S_B = 128..255, O_A = 256.., O_B = 256+D..
+// P_X (bf16) overwrites the first 64 columns of S_X and is the TMEM A operand
+// of O_X += P_X V_j; V_j is an MN-major shared-memory B operand.
+// MMA issue order per key block j (ping-pong):
+//   O_A += P_A(j-1) V_{j-1};  S_A(j) = Q_A K_j^T;  O_B += P_B(j-1) V_{j-1};  S_B(j) = Q_B K_j^T
+// so the softmax of one tile runs while the tensor pipe works on the other.
+// Because S_X(j) is issued after P_X(j-1) V_{j-1}, every MMA that touches O_X
+// has completed when S_X(j) has: the softmax warps rescale O_X in TMEM (lazily,
+// only when the row max rises by more than kRescaleThreshold) with no extra wait.
+// Softmax: base-2 online softmax in fp32 (t = s * scale * log2 e, ex2 on the
+// MUFU unit), P rounded to bf16 (RNE); epilogue o = O / l -> bf16,
+// lse = ln 2 * (m + log2 l).  Causal tiles visit key blocks 0..qt only and mask
+// only the diagonal block; sequence tails are masked by key position.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
@@ -39,126 +48,141 @@
 namespace mk {
 
 constexpr int kTile = 128;            // query rows per tile, keys per block
-constexpr int kSoftmaxThreads = 128;  // warps 0..3, one thread per query row
-constexpr int kMmaWarp = 4;
-constexpr int kLoadWarp = 5;
-constexpr int kThreads = 192;
+constexpr int kSoftmaxThreads = 128;  // per tile: one thread per query row
+constexpr int kMmaWarp = 8;
+constexpr int kLoadWarp = 9;
+constexpr int kThreads = 384;
+constexpr int kLaunchRegs = 168;      // 65536 / 384, rounded down to a multiple of 8
+constexpr uint32_t kRegsSoftmax = 208;
+constexpr uint32_t kRegsCtl = 80;
+static_assert(2 * kRegsSoftmax + kRegsCtl <= 3 * kLaunchRegs, "register split");
 constexpr int kBoxCols = 64;          // bf16 elements per 128-byte swizzle row
 constexpr int kBoxBytes = kTile * kBoxCols * 2;  // one TMA box: 128 rows x 128 B
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColS = 0;         // S buffer sb at kColS + 128 * sb
-constexpr uint32_t kColO = 256;
+constexpr uint32_t kColS = 0;         // S_X at kColS + 128 * X
+constexpr uint32_t kColO = 256;       // O_X at kColO + D * X
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: rescale O when m rises by > 2^8
+constexpr int kCuCache = 2048;        // cu_seqlens entries cached in shared memory
 
-__device__ int g_status = 0;              // MK_ERR_TIMEOUT once a wait ran out
-__device__ unsigned int g_abort_epoch = 0; // launch epoch that timed out
+__device__ int g_status = 0;               // MK_ERR_TIMEOUT once a wait ran out
+__device__ unsigned int g_abort_epoch = 0;  // launch epoch that timed out
 
 template <int D>
 struct KernelCfg {
   static_assert(D == 64 || D == 128, "head dimension 64 or 128");
   static constexpr int kStages = (D == 128) ? 2 : 4;
-  static constexpr int kHalves = D / kBoxCols;        // swizzle boxes per tile
-  static constexpr int kTileBytes = kTile * D * 2;    // one Q, K or V tile
-  static constexpr int kOffQ = 0;
-  static constexpr int kOffK = kOffQ + kTileBytes;
+  static constexpr int kHalves = D / kBoxCols;      // swizzle boxes per tile
+  static constexpr int kTileBytes = kTile * D * 2;  // one Q, K or V tile
+  static constexpr int kOffQ = 0;                   // Q_A, then Q_B
+  static constexpr int kOffK = 2 * kTileBytes;
   static constexpr int kOffV = kOffK + kStages * kTileBytes;
-  static constexpr int kOffBar = kOffV + kStages * kTileBytes;
-  static constexpr int kSmemBytes = kOffBar + 256 + 1024;  // + barriers + alignment slack
+  static constexpr int kOffCu = kOffV + kStages * kTileBytes;
+  static constexpr int kOffCtl = kOffCu + kCuCache * 4;
+  static constexpr int kSmemBytes = kOffCtl + 512 + 1024;  // + control block + alignment slack
 };
 
 struct SharedCtl {
-  uint64_t bar_q;
+  uint64_t bar_q_full[2], bar_q_empty[2];
   uint64_t bar_k_full[4], bar_k_empty[4];
   uint64_t bar_v_full[4], bar_v_empty[4];
   uint64_t bar_s_full[2], bar_p_full[2];
-  uint64_t bar_o_done;       // one phase per P_j V_j
-  uint64_t bar_o_final;      // the last P_j V_j of the tile
+  uint64_t bar_o_final[2];
   uint64_t bar_mma_drained;
   uint32_t tmem_base;
   int abort;
-  int tile_valid, tile_b, tile_qt, tile_seq_start, tile_len;
 };
-static_assert(sizeof(SharedCtl) <= 256, "control block");
+static_assert(sizeof(SharedCtl) <= 512, "control block");
 
 struct Params {
-  uint16_t *o;             // bf16 bits
+  uint16_t *o;              // bf16 bits
   float *lse;
   const int32_t *cu_seqlens;
-  int B, Hq, Hkv, S;       // S = tokens per sequence, or total tokens T (varlen)
-  int group;               // Hq / Hkv
+  int B, Hq, Hkv, S;        // S = tokens per sequence, or total tokens T (varlen)
+  int group;                // Hq / Hkv
   int causal, varlen;
-  int n_qtiles;            // fixed: ceil(S/128) ; varlen: bound on tiles per head
-  float scale_log2;        // scale * log2(e)
+  int n_pairs;              // fixed length: query-tile pairs per sequence
+  int n_units;              // fixed: exact; varlen: upper bound
+  float scale_log2;         // scale * log2(e)
   unsigned int epoch;
+};
+
+struct Unit {
+  int valid;
+  int b, hq, pair;
+  int seq_start, len;
 };
 
 __device__ __forceinline__ int clamp_tok(int x, int T) { return x < 0 ? 0 : (x > T ? T : x); }
 
-// Maps this CTA to (sequence, query tile, head).  Fixed length: causal tiles
-// are ordered longest first (largest qt first) so that the hardware's in-order
-// CTA dispatch approximates longest-processing-time scheduling.  Varlen: warp 0
-// scans cu_seqlens (clamped to [0, T], negative lengths read as 0) and finds the
-// sequence holding tile `rank` of this head.
-__device__ __forceinline__ void map_tile(const Params &p, SharedCtl *ctl, int &hq) {
-  const int idx = blockIdx.x;
+__device__ __forceinline__ int pairs_of_len(int L) { return ((L + kTile - 1) / kTile + 1) / 2; }
+
+// Maps unit index u to (sequence, query head, tile pair).  Must be called by
+// all 32 lanes of a warp (varlen uses a warp scan); every lane gets the result.
+// Fixed length: units are ordered by pair, heaviest first when causal, so that
+// the static round-robin over CTAs approximates longest-processing-time order;
+// consecutive units share a K/V head (GQA groups are contiguous).  Varlen: unit
+// u is pair `u / Hq` of head u % Hq in sequence order; cu_seqlens entries are
+// clamped to [0, T] and negative lengths read as zero.
+__device__ __forceinline__ Unit map_unit(const Params &p, const int *cu_smem, int u) {
+  Unit w;
   if (!p.varlen) {
     const int per_level = p.B * p.Hq;
-    const int level = idx / per_level;
-    const int rem = idx - level * per_level;
-    hq = rem % p.Hq;
-    if (threadIdx.x == 0) {
-      const int b = rem / p.Hq;
-      ctl->tile_valid = 1;
-      ctl->tile_b = b;
-      ctl->tile_qt = p.causal ? (p.n_qtiles - 1 - level) : level;
-      ctl->tile_seq_start = b * p.S;
-      ctl->tile_len = p.S;
-    }
-    return;
+    const int level = u / per_level;
+    const int rem = u - level * per_level;
+    w.valid = u < p.n_units;
+    w.hq = rem % p.Hq;
+    w.b = rem / p.Hq;
+    w.pair = p.causal ? (p.n_pairs - 1 - level) : level;
+    w.seq_start = w.b * p.S;
+    w.len = p.S;
+    return w;
   }
-  hq = idx % p.Hq;
-  if (threadIdx.x < 32) {
-    const int rank = idx / p.Hq;
-    const int lane = threadIdx.x;
-    const int T = p.S;
-    int carry = 0;
-    int found = 0, f_b = 0, f_qt = 0, f_s0 = 0, f_len = 0;
-    for (int base = 0; base < p.B && !found; base += 32) {
-      const int b = base + lane;
-      int s0 = 0, s1 = 0, nt = 0;
-      if (b < p.B) {
-        s0 = clamp_tok(p.cu_seqlens[b], T);
-        s1 = clamp_tok(p.cu_seqlens[b + 1], T);
-        if (s1 < s0) s1 = s0;
-        nt = (s1 - s0 + kTile - 1) / kTile;
-      }
-      int incl = nt;
+  const int lane = lane_id();
+  const int rank = u / p.Hq;
+  const int T = p.S;
+  w.hq = u % p.Hq;
+  w.valid = 0;
+  w.b = w.pair = w.seq_start = w.len = 0;
+  int carry = 0;
+  for (int base = 0; base < p.B; base += 32) {
+    const int b = base + lane;
+    int s0 = 0, s1 = 0, np = 0;
+    if (b < p.B) {
+      s0 = clamp_tok(b < kCuCache ? cu_smem[b] : p.cu_seqlens[b], T);
+      s1 = clamp_tok(b + 1 < kCuCache ? cu_smem[b + 1] : p.cu_seqlens[b + 1], T);
+      if (s1 < s0) s1 = s0;
+      np = pairs_of_len(s1 - s0);
+    }
+    int incl = np;
 #pragma unroll
-      for (int off = 1; off < 32; off <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, incl, off);
-        if (lane >= off) incl += y;
-      }
-      const int excl = incl - nt;
-      const bool mine = (b < p.B) && rank >= carry + excl && rank < carry + incl;
-      const unsigned m = __ballot_sync(0xffffffffu, mine);
-      if (m) {
-        const int src = __ffs(m) - 1;
-        f_b = base + src;
-        f_qt = rank - carry - __shfl_sync(0xffffffffu, excl, src);
-        f_s0 = __shfl_sync(0xffffffffu, s0, src);
-        f_len = __shfl_sync(0xffffffffu, s1 - s0, src);
-        found = 1;
-      }
-      carry += __shfl_sync(0xffffffffu, incl, 31);
+    for (int off = 1; off < 32; off <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += y;
     }
-    if (lane == 0) {
-      ctl->tile_valid = found;
-      ctl->tile_b = f_b;
-      ctl->tile_qt = f_qt;
-      ctl->tile_seq_start = f_s0;
-      ctl->tile_len = f_len;
+    const int excl = incl - np;
+    const bool mine = (b < p.B) && rank >= carry + excl && rank < carry + incl;
+    const unsigned m = __ballot_sync(0xffffffffu, mine);
+    if (m) {
+      const int src = __ffs(m) - 1;
+      w.valid = 1;
+      w.b = base + src;
+      w.pair = rank - carry - __shfl_sync(0xffffffffu, excl, src);
+      w.seq_start = __shfl_sync(0xffffffffu, s0, src);
+      w.len = __shfl_sync(0xffffffffu, s1 - s0, src);
+      break;
     }
+    carry += __shfl_sync(0xffffffffu, incl, 31);
   }
+  return w;
+}
+
+// Key blocks visited by tile X (0 = A, 1 = B) of a unit; 0 if the tile lies
+// past the end of the sequence.
+__device__ __forceinline__ int tile_blocks(const Params &p, const Unit &w, int X) {
+  const int qt = 2 * w.pair + X;
+  if (qt * kTile >= w.len) return 0;
+  const int n_kb = (w.len + kTile - 1) / kTile;
+  return p.causal ? min(qt + 1, n_kb) : n_kb;
 }
 
 // Bounded wait that ignores the abort flag: used only at teardown to let
@@ -182,36 +206,35 @@ __global__ void __launch_bounds__(kThreads, 1)
   // 1024-byte alignment for the 128-byte-swizzle atoms.
   const uint32_t raw_addr = smem_addr(smem_raw);
   uint8_t *smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);
-  SharedCtl *ctl = reinterpret_cast<SharedCtl *>(smem + C::kOffBar);
+  SharedCtl *ctl = reinterpret_cast<SharedCtl *>(smem + C::kOffCtl);
+  int *cu_smem = reinterpret_cast<int *>(smem + C::kOffCu);
   const uint32_t sQ = smem_addr(smem + C::kOffQ);
   const uint32_t sK = smem_addr(smem + C::kOffK);
   const uint32_t sV = smem_addr(smem + C::kOffV);
-
   const int warp = threadIdx.x / 32;
-  int hq = 0;
-  map_tile(p, ctl, hq);
 
+  if (p.varlen) {
+    const int n = min(p.B + 1, kCuCache);
+    for (int i = threadIdx.x; i < n; i += kThreads) cu_smem[i] = p.cu_seqlens[i];
+  }
   if (threadIdx.x == 0) {
-    mbar_init(&ctl->bar_q, 1);
+    for (int x = 0; x < 2; ++x) {
+      mbar_init(&ctl->bar_q_full[x], 1);
+      mbar_init(&ctl->bar_q_empty[x], 1);
+      mbar_init(&ctl->bar_s_full[x], 1);
+      mbar_init(&ctl->bar_p_full[x], kSoftmaxThreads);
+      mbar_init(&ctl->bar_o_final[x], 1);
+    }
     for (int s = 0; s < NS; ++s) {
       mbar_init(&ctl->bar_k_full[s], 1);
       mbar_init(&ctl->bar_k_empty[s], 1);
       mbar_init(&ctl->bar_v_full[s], 1);
       mbar_init(&ctl->bar_v_empty[s], 1);
     }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(&ctl->bar_s_full[b], 1);
-      mbar_init(&ctl->bar_p_full[b], kSoftmaxThreads);
-    }
-    mbar_init(&ctl->bar_o_done, 1);
-    mbar_init(&ctl->bar_o_final, 1);
     mbar_init(&ctl->bar_mma_drained, 1);
     ctl->abort = 0;
     fence_mbar_init();
   }
-  __syncthreads();
-  if (!ctl->tile_valid) return;  // uniform: varlen CTAs beyond the last tile
-
   if (warp == kMmaWarp) {
     tmem_alloc(&ctl->tmem_base, kTmemCols);
     tmem_relinquish_alloc_permit();
@@ -220,254 +243,389 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after_sync();
   const uint32_t tmem = ctl->tmem_base;
-
-  const int qt = ctl->tile_qt;
-  const int seq_start = ctl->tile_seq_start;
-  const int L = ctl->tile_len;
-  const int hkv = hq / p.group;
-  const int n_kblocks_seq = (L + kTile - 1) / kTile;
-  const int nblk = p.causal ? min(qt + 1, n_kblocks_seq) : n_kblocks_seq;
   volatile int *abort = &ctl->abort;
 
-  if (warp == kLoadWarp) {
-    // ------------------------------------------------------------ producer
-    if (lane_id() == 0) {
-      tma_prefetch_desc(&tm_q);
-      tma_prefetch_desc(&tm_k);
-      tma_prefetch_desc(&tm_v);
-      const uint64_t pol_q = l2_policy_evict_first();
-      const uint64_t pol_kv = l2_policy_evict_last();
-      mbar_arrive_expect_tx(&ctl->bar_q, C::kTileBytes);
-      for (int h = 0; h < C::kHalves; ++h)
-        tma_load_3d(smem + C::kOffQ + h * kBoxBytes, &tm_q, &ctl->bar_q, h * kBoxCols, hq,
-                    seq_start + qt * kTile, pol_q);
-      int issued = 0;
-      for (int j = 0; j < nblk; ++j) {
-        const int s = j % NS;
-        const uint32_t ph = (j / NS) & 1;
-        if (!mbar_wait(&ctl->bar_k_empty[s], ph ^ 1, abort)) break;
-        mbar_arrive_expect_tx(&ctl->bar_k_full[s], C::kTileBytes);
-        for (int h = 0; h < C::kHalves; ++h)
-          tma_load_3d(smem + C::kOffK + s * C::kTileBytes + h * kBoxBytes, &tm_k,
-                      &ctl->bar_k_full[s], h * kBoxCols, hkv, seq_start + j * kTile, pol_kv);
-        if (!mbar_wait(&ctl->bar_v_empty[s], ph ^ 1, abort)) {
-          issued = j * 2 + 1;
-          break;
+  if (warp >= 8) {
+    // Third warpgroup: producer, MMA issuer and two idle warps.  All four
+    // warps give registers back at this one instruction.
+    setmaxnreg_dec<kRegsCtl>();
+    // The producer and MMA warps run their loops and waits with all 32 lanes
+    // converged; one lane chosen by elect.sync issues each TMA / tcgen05
+    // instruction.  Keeping the warp converged lets the unit bookkeeping and
+    // the matrix descriptors live in warp-uniform registers, so consecutive
+    // tcgen05.mma issue back to back.
+    if (warp == kLoadWarp) {
+      // ---------------------------------------------------------- producer
+      uint64_t pol_q = 0, pol_kv = 0;
+      if (elect_one()) {
+        tma_prefetch_desc(&tm_q);
+        tma_prefetch_desc(&tm_k);
+        tma_prefetch_desc(&tm_v);
+      }
+      pol_q = l2_policy_evict_first();
+      pol_kv = l2_policy_evict_last();
+      uint32_t q_iter = 0, kv_iter = 0;
+      uint32_t k_issued = 0, v_issued = 0;  // loads issued, for the drain below
+      bool ok = true;
+      for (int u = blockIdx.x; ok && u < p.n_units; u += gridDim.x) {
+        const Unit w = map_unit(p, cu_smem, u);
+        if (!w.valid) continue;
+        const int hkv = w.hq / p.group;
+        const int n_blk = max(tile_blocks(p, w, 0), tile_blocks(p, w, 1));
+        for (int x = 0; x < 2; ++x) {
+          ok = __all_sync(0xffffffffu, mbar_wait(&ctl->bar_q_empty[x], (q_iter & 1) ^ 1, abort));
+          if (!ok) break;
+          if (elect_one()) {
+            mbar_arrive_expect_tx(&ctl->bar_q_full[x], C::kTileBytes);
+#pragma unroll
+            for (int h = 0; h < C::kHalves; ++h)
+              tma_load_3d(smem + C::kOffQ + x * C::kTileBytes + h * kBoxBytes, &tm_q,
+                          &ctl->bar_q_full[x], h * kBoxCols, w.hq,
+                          w.seq_start + (2 * w.pair + x) * kTile, pol_q);
+          }
+          __syncwarp();
         }
-        mbar_arrive_expect_tx(&ctl->bar_v_full[s], C::kTileBytes);
-        for (int h = 0; h < C::kHalves; ++h)
-          tma_load_3d(smem + C::kOffV + s * C::kTileBytes + h * kBoxBytes, &tm_v,
-                      &ctl->bar_v_full[s], h * kBoxCols, hkv, seq_start + j * kTile, pol_kv);
-        issued = j * 2 + 2;
+        if (!ok) break;
+        ++q_iter;
+        for (int j = 0; j < n_blk; ++j, ++kv_iter) {
+          const int s = kv_iter % NS;
+          const uint32_t ph = (kv_iter / NS) & 1;
+          ok = __all_sync(0xffffffffu, mbar_wait(&ctl->bar_k_empty[s], ph ^ 1, abort));
+          if (!ok) break;
+          if (elect_one()) {
+            mbar_arrive_expect_tx(&ctl->bar_k_full[s], C::kTileBytes);
+#pragma unroll
+            for (int h = 0; h < C::kHalves; ++h)
+              tma_load_3d(smem + C::kOffK + s * C::kTileBytes + h * kBoxBytes, &tm_k,
+                          &ctl->bar_k_full[s], h * kBoxCols, hkv, w.seq_start + j * kTile,
+                          pol_kv);
+          }
+          __syncwarp();
+          k_issued = kv_iter + 1;
+          ok = __all_sync(0xffffffffu, mbar_wait(&ctl->bar_v_empty[s], ph ^ 1, abort));
+          if (!ok) break;
+          if (elect_one()) {
+            mbar_arrive_expect_tx(&ctl->bar_v_full[s], C::kTileBytes);
+#pragma unroll
+            for (int h = 0; h < C::kHalves; ++h)
+              tma_load_3d(smem + C::kOffV + s * C::kTileBytes + h * kBoxBytes, &tm_v,
+                          &ctl->bar_v_full[s], h * kBoxCols, hkv, w.seq_start + j * kTile,
+                          pol_kv);
+          }
+          __syncwarp();
+          v_issued = kv_iter + 1;
+        }
       }
-      // Teardown: every load issued must land before the CTA exits.
-      drain_wait(&ctl->bar_q, 0);
-      for (int n = (issued > 2 * NS ? issued - 2 * NS : 0); n < issued; ++n) {
-        const int j = n / 2, s = j % NS;
-        const uint32_t ph = (j / NS) & 1;
-        drain_wait((n & 1) ? &ctl->bar_v_full[s] : &ctl->bar_k_full[s], ph);
-      }
-    }
-  } else if (warp == kMmaWarp) {
-    // ------------------------------------------------------------ MMA issuer
-    if (lane_id() == 0) {
+      // Teardown: every load issued must land before the CTA exits.  For each
+      // stage the last issued phase is waited for (earlier phases precede it).
+      if (q_iter > 0)
+        for (int x = 0; x < 2; ++x) drain_wait(&ctl->bar_q_full[x], (q_iter - 1) & 1);
+      for (uint32_t n = (k_issued > (uint32_t)NS ? k_issued - NS : 0); n < k_issued; ++n)
+        drain_wait(&ctl->bar_k_full[n % NS], (n / NS) & 1);
+      for (uint32_t n = (v_issued > (uint32_t)NS ? v_issued - NS : 0); n < v_issued; ++n)
+        drain_wait(&ctl->bar_v_full[n % NS], (n / NS) & 1);
+    } else if (warp == kMmaWarp) {
+      // ---------------------------------------------------------- MMA issuer
       constexpr uint32_t idesc_qk = idesc_bf16_f32(kTile, kTile, false, false);
       constexpr uint32_t idesc_pv = idesc_bf16_f32(kTile, D, false, true);
-      bool ok = mbar_wait(&ctl->bar_q, 0, abort);
-      auto issue_pv = [&](int i) -> bool {
-        const int sb = i & 1, s = i % NS;
-        const uint32_t ph = (i / NS) & 1;
-        if (!mbar_wait(&ctl->bar_p_full[sb], (i >> 1) & 1, abort)) return false;
-        if (!mbar_wait(&ctl->bar_v_full[s], ph, abort)) return false;
-        tc_fence_after_sync();
-        const uint32_t v_base = sV + s * C::kTileBytes;
-#pragma unroll
-        for (int kk = 0; kk < kTile / 16; ++kk) {
-          // V as the B operand of P V: N = head dim (contiguous, MN-major),
-          // K = keys.  8-key groups are 1024 B apart (SBO); 64-column chunks
-          // of the head dimension are one TMA box (16 KB) apart (LBO).  With
-          // D = 64 there is one chunk and the LBO field is not used.
-          constexpr uint32_t kVLbo = (D > kBoxCols) ? kBoxBytes : 1024;
-          const uint64_t bdesc = sdesc_sw128(v_base + kk * 16 * 128, kVLbo, 1024);
-          umma_ts(tmem + kColO, tmem + kColS + sb * 128 + kk * 8, bdesc, idesc_pv,
-                  (i > 0 || kk > 0) ? 1u : 0u);
-        }
-        umma_commit(&ctl->bar_v_empty[s]);
-        umma_commit(&ctl->bar_o_done);
-        if (i == nblk - 1) umma_commit(&ctl->bar_o_final);
-        return true;
-      };
-      for (int j = 0; ok && j < nblk; ++j) {
-        const int s = j % NS, sb = j & 1;
-        const uint32_t ph = (j / NS) & 1;
-        if (!mbar_wait(&ctl->bar_k_full[s], ph, abort)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after_sync();
-        const uint32_t k_base = sK + s * C::kTileBytes;
+      // Q and K are K-major (head dim contiguous); 16 bf16 = 32 B per MMA step
+      // inside a 128-byte swizzle row, 8-row groups 1024 B apart.  V is the
+      // MN-major B operand of P V: 8-key groups 1024 B apart (SBO), 64-column
+      // chunks of the head dimension one TMA box apart (LBO, unused at D = 64).
+      // The descriptor's address field is addr >> 4, so stepping the start
+      // address by b bytes adds b >> 4 to the descriptor.
+      constexpr uint32_t kVLbo = (D > kBoxCols) ? kBoxBytes : 1024;
+      const uint64_t dq0 = sdesc_sw128(sQ, 16, 1024);
+      const uint64_t dk0 = sdesc_sw128(sK, 16, 1024);
+      const uint64_t dv0 = sdesc_sw128(sV, kVLbo, 1024);
+      constexpr uint64_t kTileStep = C::kTileBytes >> 4;
+      uint32_t q_iter = 0, kv_iter = 0;
+      uint32_t p_cnt[2] = {0, 0};
+      bool ok = true;
+
+      // S_X = Q_X K^T for the K tile in stage s (elected lane only).
+      auto issue_s = [&](int x, int s) {
+        const uint64_t a0 = dq0 + x * kTileStep;
+        const uint64_t b0 = dk0 + s * kTileStep;
+        const uint32_t d_tmem = tmem + kColS + x * 128;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          // Q and K are K-major (head dim contiguous); 16 bf16 = 32 B per MMA
-          // step inside a 128-byte swizzle row; 8-row groups 1024 B apart.
-          const uint32_t off = (kk / 4) * kBoxBytes + (kk % 4) * 32;
-          const uint64_t adesc = sdesc_sw128(sQ + off, 16, 1024);
-          const uint64_t bdesc = sdesc_sw128(k_base + off, 16, 1024);
-          umma_ss(tmem + kColS + sb * 128, adesc, bdesc, idesc_qk, kk > 0 ? 1u : 0u);
+          const uint32_t off = ((kk >> 2) * kBoxBytes + (kk & 3) * 32) >> 4;
+          umma_ss(d_tmem, a0 + off, b0 + off, idesc_qk, kk > 0 ? 1u : 0u);
         }
-        umma_commit(&ctl->bar_s_full[sb]);
-        umma_commit(&ctl->bar_k_empty[s]);
-        if (j > 0 && !issue_pv(j - 1)) ok = false;
+        umma_commit(&ctl->bar_s_full[x]);
+      };
+      // O_X (+)= P_X V for the V tile in stage s (elected lane only).
+      auto issue_pv = [&](int x, int s, bool first) {
+        const uint64_t b0 = dv0 + s * kTileStep;
+        const uint32_t d_tmem = tmem + kColO + x * D;
+        const uint32_t a_tmem = tmem + kColS + x * 128;
+#pragma unroll
+        for (int kk = 0; kk < kTile / 16; ++kk)
+          umma_ts(d_tmem, a_tmem + kk * 8, b0 + (uint64_t)(kk * 128), idesc_pv,
+                  (!first || kk > 0) ? 1u : 0u);
+      };
+
+      for (int u = blockIdx.x; ok && u < p.n_units; u += gridDim.x) {
+        const Unit w = map_unit(p, cu_smem, u);
+        if (!w.valid) continue;
+        const int n0 = tile_blocks(p, w, 0);
+        const int n1 = tile_blocks(p, w, 1);
+        const int n_blk = max(n0, n1);
+        for (int x = 0; x < 2 && ok; ++x)
+          ok = __all_sync(0xffffffffu, mbar_wait(&ctl->bar_q_full[x], q_iter & 1, abort));
+        // j = 0: S_A(0), S_B(0)
+        int s_cur = kv_iter % NS;
+        if (ok)
+          ok = __all_sync(0xffffffffu,
+                          mbar_wait(&ctl->bar_k_full[s_cur], (kv_iter / NS) & 1, abort));
+        if (ok) {
+          tc_fence_after_sync();
+          if (elect_one()) {
+            if (n0 > 0) issue_s(0, s_cur);
+            if (n0 <= 1) umma_commit(&ctl->bar_q_empty[0]);  // Q_A no longer read
+            if (n1 > 0) issue_s(1, s_cur);
+            if (n1 <= 1) umma_commit(&ctl->bar_q_empty[1]);
+            umma_commit(&ctl->bar_k_empty[s_cur]);
+          }
+          __syncwarp();
+        }
+        for (int j = 1; ok && j <= n_blk; ++j) {
+          const uint32_t it_prev = kv_iter + j - 1;
+          const int s_prev = it_prev % NS;
+          const bool has_next = j < n_blk;
+          const uint32_t it_cur = kv_iter + j;
+          s_cur = it_cur % NS;
+          ok = __all_sync(0xffffffffu,
+                          mbar_wait(&ctl->bar_v_full[s_prev], (it_prev / NS) & 1, abort));
+          if (ok && has_next)
+            ok = __all_sync(0xffffffffu,
+                            mbar_wait(&ctl->bar_k_full[s_cur], (it_cur / NS) & 1, abort));
+#pragma unroll
+          for (int x = 0; x < 2; ++x) {
+            const int nx = x == 0 ? n0 : n1;
+            if (ok && j - 1 < nx) {
+              ok = __all_sync(0xffffffffu,
+                              mbar_wait(&ctl->bar_p_full[x], p_cnt[x] & 1, abort));
+              ++p_cnt[x];
+            }
+            if (!ok) break;
+            tc_fence_after_sync();
+            if (elect_one()) {
+              if (j - 1 < nx) {
+                issue_pv(x, s_prev, j == 1);
+                if (j - 1 == nx - 1) umma_commit(&ctl->bar_o_final[x]);
+              }
+              if (has_next && j < nx) {
+                issue_s(x, s_cur);
+                if (j == nx - 1) umma_commit(&ctl->bar_q_empty[x]);
+              }
+            }
+            __syncwarp();
+          }
+          if (!ok) break;
+          if (elect_one()) {
+            umma_commit(&ctl->bar_v_empty[s_prev]);
+            if (has_next) umma_commit(&ctl->bar_k_empty[s_cur]);
+          }
+          __syncwarp();
+        }
+        kv_iter += n_blk;
+        ++q_iter;
       }
-      if (ok) issue_pv(nblk - 1);
-      // Teardown: all MMAs issued by this thread complete before TMEM is freed.
-      umma_commit(&ctl->bar_mma_drained);
+      // Teardown: all MMAs issued by this warp complete before TMEM is freed.
+      if (elect_one()) umma_commit(&ctl->bar_mma_drained);
+      __syncwarp();
       drain_wait(&ctl->bar_mma_drained, 0);
     }
   } else {
     // ------------------------------------------------------------ softmax
-    const int r = threadIdx.x;  // query row within the tile == TMEM lane
-    const uint32_t t_row = tmem + ((uint32_t)(warp * 32) << 16);
-    const int qpos = qt * kTile + r;
-    const bool row_valid = qpos < L;
-    const int key_limit = p.causal ? min(L, qpos + 1) : L;  // keys [0, key_limit) visible
+    // Both softmax warpgroups take their larger register budget here.
+    setmaxnreg_inc<kRegsSoftmax>();
+    const int X = warp / 4;                       // tile of this warpgroup
+    const int r = threadIdx.x % kSoftmaxThreads;  // row within the tile == TMEM lane
+    const uint32_t t_row = tmem + ((uint32_t)((warp % 4) * 32) << 16);
+    const uint32_t t_s = t_row + kColS + X * 128;
+    const uint32_t t_o = t_row + kColO + X * D;
     const float c2 = p.scale_log2;
-    float m_run = -INFINITY;  // running row max, base-2 units
-    float l_run = 0.f;        // running row sum relative to m_run
+    const bool neg_scale = c2 < 0.f;
+    const float mask_val = neg_scale ? INFINITY : -INFINITY;
+    uint32_t s_cnt = 0, o_cnt = 0;
     bool ok = true;
 
-    for (int j = 0; j < nblk; ++j) {
-      const int sb = j & 1;
-      ok = mbar_wait(&ctl->bar_s_full[sb], (j >> 1) & 1, abort);
-      if (!__all_sync(0xffffffffu, ok)) {
-        ok = false;
-        *abort = 1;
-        break;
-      }
-      tc_fence_after_sync();
-      float t[kTile];
-      {
-        uint32_t raw[4][32];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) tmem_ld_32x32b_x32(t_row + kColS + sb * 128 + c * 32, raw[c]);
-        tmem_ld_wait();
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          reg_fence(raw[c]);
-#pragma unroll
-          for (int e = 0; e < 32; ++e) t[c * 32 + e] = __uint_as_float(raw[c][e]) * c2;
-        }
-      }
-      const bool needs_mask = (j * kTile + kTile > L) || (p.causal && j == qt);
-      if (needs_mask) {
-        const int lim = key_limit - j * kTile;
-#pragma unroll
-        for (int c = 0; c < kTile; ++c) t[c] = (c < lim) ? t[c] : -INFINITY;
-      }
-      float mx0 = t[0], mx1 = t[1], mx2 = t[2], mx3 = t[3];
-#pragma unroll
-      for (int c = 4; c < kTile; c += 4) {
-        mx0 = fmaxf(mx0, t[c]);
-        mx1 = fmaxf(mx1, t[c + 1]);
-        mx2 = fmaxf(mx2, t[c + 2]);
-        mx3 = fmaxf(mx3, t[c + 3]);
-      }
-      const float m_blk = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3));
-      const float m_new = fmaxf(m_run, m_blk);
-      // Lazy rescaling: keep the old reference max unless the new one exceeds
-      // it by more than the threshold.  Exact either way, because O and l
-      // always share the same reference max.
-      const bool rescale = m_new > m_run + kRescaleThreshold;
-      float alpha = 1.f;
-      if (rescale) {
-        alpha = ex2_approx(m_run - m_new);  // 0 when m_run = -inf
-        l_run *= alpha;
-        m_run = m_new;
-      }
-      if (j > 0 && __any_sync(0xffffffffu, rescale)) {
-        // O holds blocks 0..j-1 only once P_{j-1} V_{j-1} has completed.
-        ok = mbar_wait(&ctl->bar_o_done, (j - 1) & 1, abort);
+    for (int u = blockIdx.x; ok && u < p.n_units; u += gridDim.x) {
+      const Unit w = map_unit(p, cu_smem, u);
+      if (!w.valid) continue;
+      const int n_blk = tile_blocks(p, w, X);
+      if (n_blk == 0) continue;
+      const int qt = 2 * w.pair + X;
+      const int qpos = qt * kTile + r;
+      const bool row_valid = qpos < w.len;
+      const int key_limit = p.causal ? min(w.len, qpos + 1) : w.len;  // keys [0, limit)
+      float m_run = -INFINITY;  // running row max, base-2 units
+      float l_run = 0.f;        // running row sum relative to m_run
+
+      for (int j = 0; j < n_blk; ++j) {
+        ok = mbar_wait(&ctl->bar_s_full[X], s_cnt & 1, abort);
+        ++s_cnt;
         if (!__all_sync(0xffffffffu, ok)) {
           ok = false;
-          *abort = 1;
           break;
         }
         tc_fence_after_sync();
+        const bool needs_mask = (j * kTile + kTile > w.len) || (p.causal && j == qt);
+        const int lim = key_limit - j * kTile;
+        // s = raw S_X(j) row.  Hidden keys take the value that loses the
+        // max (min when scale < 0), and get p = 0 after the exponential, so the
+        // mask holds for every sign of the scale, zero included.
+        auto load_scores = [&](float (&s)[kTile]) {
+          uint32_t raw[4][32];
 #pragma unroll
-        for (int c = 0; c < D / 32; ++c) {
-          uint32_t o_raw[32];
-          tmem_ld_32x32b_x32(t_row + kColO + c * 32, o_raw);
+          for (int c = 0; c < 4; ++c) tmem_ld_32x32b_x32(t_s + c * 32, raw[c]);
           tmem_ld_wait();
-          reg_fence(o_raw);
 #pragma unroll
-          for (int e = 0; e < 32; ++e)
-            o_raw[e] = __float_as_uint(__uint_as_float(o_raw[e]) * alpha);
-          tmem_st_32x32b_x32(t_row + kColO + c * 32, o_raw);
+          for (int c = 0; c < 4; ++c) {
+            reg_fence(raw[c]);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) s[c * 32 + e] = __uint_as_float(raw[c][e]);
+          }
+          if (needs_mask) {
+#pragma unroll
+            for (int c = 0; c < kTile; ++c) s[c] = (c < lim) ? s[c] : mask_val;
+          }
+        };
+        float s[kTile];
+        load_scores(s);
+        // Row max of t = s * c2 (base-2 units) = c2 * (max s), or c2 * (min s)
+        // when c2 < 0.
+        float mx0, mx1, mx2, mx3;
+        if (!neg_scale) {
+          mx0 = fmaxf(s[0], s[1]);
+          mx1 = fmaxf(s[2], s[3]);
+          mx2 = fmaxf(s[4], s[5]);
+          mx3 = fmaxf(s[6], s[7]);
+#pragma unroll
+          for (int c = 8; c < kTile; c += 8) {
+            mx0 = fmax3(mx0, s[c], s[c + 1]);
+            mx1 = fmax3(mx1, s[c + 2], s[c + 3]);
+            mx2 = fmax3(mx2, s[c + 4], s[c + 5]);
+            mx3 = fmax3(mx3, s[c + 6], s[c + 7]);
+          }
+          mx0 = fmaxf(fmax3(mx0, mx1, mx2), mx3);
+        } else {
+          mx0 = fminf(s[0], s[1]);
+          mx1 = fminf(s[2], s[3]);
+          mx2 = fminf(s[4], s[5]);
+          mx3 = fminf(s[6], s[7]);
+#pragma unroll
+          for (int c = 8; c < kTile; c += 8) {
+            mx0 = fmin3(mx0, s[c], s[c + 1]);
+            mx1 = fmin3(mx1, s[c + 2], s[c + 3]);
+            mx2 = fmin3(mx2, s[c + 4], s[c + 5]);
+            mx3 = fmin3(mx3, s[c + 6], s[c + 7]);
+          }
+          mx0 = fminf(fmin3(mx0, mx1, mx2), mx3);
         }
-        tmem_st_wait();
-      }
-      const float m_use = (m_run == -INFINITY) ? 0.f : m_run;
-      float sum0 = 0.f, sum1 = 0.f, sum2 = 0.f, sum3 = 0.f;
-      uint32_t pk[2][32];
+        const float m_new = fmaxf(m_run, mx0 * c2);  // fmaxf drops a NaN (0 * inf)
+        // Lazy rescaling: keep the old reference max unless the new one exceeds
+        // it by more than the threshold.  Exact either way, because O and l
+        // always share the same reference max.
+        const bool rescale = m_new > m_run + kRescaleThreshold;
+        float alpha = 1.f;
+        if (rescale) {
+          alpha = ex2_approx(m_run - m_new);  // 0 when m_run = -inf
+          l_run *= alpha;
+          m_run = m_new;
+        }
+        if (j > 0 && __any_sync(0xffffffffu, rescale)) {
+          // O_X already holds blocks 0..j-1: P_X(j-1) V_{j-1} was issued before
+          // S_X(j), and S_X(j) has completed.  The scores are read again
+          // afterwards rather than kept live across this (rare) step.
 #pragma unroll
-      for (int c = 0; c < kTile; c += 4) {
-        const float p0 = ex2_approx(t[c] - m_use);
-        const float p1 = ex2_approx(t[c + 1] - m_use);
-        const float p2 = ex2_approx(t[c + 2] - m_use);
-        const float p3 = ex2_approx(t[c + 3] - m_use);
-        sum0 += p0;
-        sum1 += p1;
-        sum2 += p2;
-        sum3 += p3;
-        pk[c / 64][(c % 64) / 2] = pack_bf16x2(p0, p1);
-        pk[c / 64][(c % 64) / 2 + 1] = pack_bf16x2(p2, p3);
+          for (int c = 0; c < D / 32; ++c) {
+            uint32_t o_raw[32];
+            tmem_ld_32x32b_x32(t_o + c * 32, o_raw);
+            tmem_ld_wait();
+            reg_fence(o_raw);
+#pragma unroll
+            for (int e = 0; e < 32; ++e)
+              o_raw[e] = __float_as_uint(__uint_as_float(o_raw[e]) * alpha);
+            tmem_st_32x32b_x32(t_o + c * 32, o_raw);
+          }
+          tmem_st_wait();
+          load_scores(s);
+        }
+        // p = 2^(s * c2 - m), one packed FMA per pair of keys.
+        const float neg_m = (m_run == -INFINITY) ? 0.f : -m_run;
+        float sum0 = 0.f, sum1 = 0.f, sum2 = 0.f, sum3 = 0.f;
+        uint32_t pk[2][32];
+#pragma unroll
+        for (int c = 0; c < kTile; c += 4) {
+          float a0, a1, a2, a3;
+          ffma2_bcast(a0, a1, s[c], s[c + 1], c2, neg_m);
+          ffma2_bcast(a2, a3, s[c + 2], s[c + 3], c2, neg_m);
+          float p0 = ex2_approx(a0), p1 = ex2_approx(a1);
+          float p2 = ex2_approx(a2), p3 = ex2_approx(a3);
+          if (needs_mask) {
+            p0 = (c < lim) ? p0 : 0.f;
+            p1 = (c + 1 < lim) ? p1 : 0.f;
+            p2 = (c + 2 < lim) ? p2 : 0.f;
+            p3 = (c + 3 < lim) ? p3 : 0.f;
+          }
+          fadd2_acc(sum0, sum1, p0, p1);
+          fadd2_acc(sum2, sum3, p2, p3);
+          pk[c / 64][(c % 64) / 2] = pack_bf16x2(p0, p1);
+          pk[c / 64][(c % 64) / 2 + 1] = pack_bf16x2(p2, p3);
+        }
+        l_run += (sum0 + sum1) + (sum2 + sum3);
+        // P_X(j) (bf16, 64 columns) overwrites the first half of S_X(j).
+        tmem_st_32x32b_x32(t_s, pk[0]);
+        tmem_st_32x32b_x32(t_s + 32, pk[1]);
+        tmem_st_wait();
+        tc_fence_before_sync();
+        mbar_arrive(&ctl->bar_p_full[X]);
       }
-      l_run += (sum0 + sum1) + (sum2 + sum3);
-      // P_j (bf16, 64 columns) overwrites the first half of S_j.
-      tmem_st_32x32b_x32(t_row + kColS + sb * 128, pk[0]);
-      tmem_st_32x32b_x32(t_row + kColS + sb * 128 + 32, pk[1]);
-      tmem_st_wait();
-      tc_fence_before_sync();
-      mbar_arrive(&ctl->bar_p_full[sb]);
-    }
+      if (!ok) break;
 
-    // ------------------------------------------------------------ epilogue
-    if (ok) {
-      // A barrier of its own: bar_o_done may still be two phases short here.
-      ok = mbar_wait(&ctl->bar_o_final, 0, abort);
-      ok = __all_sync(0xffffffffu, ok);
-    }
-    if (ok) {
+      // ---------------------------------------------------------- epilogue
+      ok = mbar_wait(&ctl->bar_o_final[X], o_cnt & 1, abort);
+      ++o_cnt;
+      if (!__all_sync(0xffffffffu, ok)) {
+        ok = false;
+        break;
+      }
       tc_fence_after_sync();
       const float inv_l = 1.f / l_run;
-      const int64_t tok = (int64_t)seq_start + qpos;
-      uint4 *dst = reinterpret_cast<uint4 *>(p.o + (tok * p.Hq + hq) * (int64_t)D);
+      const int64_t tok = (int64_t)w.seq_start + qpos;
+      uint4 *dst = reinterpret_cast<uint4 *>(p.o + (tok * p.Hq + w.hq) * (int64_t)D);
 #pragma unroll
       for (int c = 0; c < D / 32; ++c) {
         uint32_t o_raw[32];
-        tmem_ld_32x32b_x32(t_row + kColO + c * 32, o_raw);
+        tmem_ld_32x32b_x32(t_o + c * 32, o_raw);
         tmem_ld_wait();
         reg_fence(o_raw);
-        uint32_t w[16];
+        uint32_t v[16];
 #pragma unroll
         for (int e = 0; e < 16; ++e)
-          w[e] = pack_bf16x2(__uint_as_float(o_raw[2 * e]) * inv_l,
+          v[e] = pack_bf16x2(__uint_as_float(o_raw[2 * e]) * inv_l,
                              __uint_as_float(o_raw[2 * e + 1]) * inv_l);
         if (row_valid) {
 #pragma unroll
           for (int e = 0; e < 4; ++e)
-            dst[c * 4 + e] = make_uint4(w[4 * e], w[4 * e + 1], w[4 * e + 2], w[4 * e + 3]);
+            dst[c * 4 + e] = make_uint4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
         }
       }
+      // O_X has been read: the next unit's first P_X V (which overwrites O_X)
+      // is issued only after this warpgroup produces that unit's P_X(0).
+      tc_fence_before_sync();
       if (row_valid) {
         const float lse = (m_run + log2f(l_run)) * 0.69314718055994530942f;
-        const int64_t li = p.varlen ? (int64_t)hq * p.S + tok
-                                    : ((int64_t)ctl->tile_b * p.Hq + hq) * p.S + qpos;
+        const int64_t li = p.varlen ? (int64_t)w.hq * p.S + tok
+                                    : ((int64_t)w.b * p.Hq + w.hq) * p.S + qpos;
         p.lse[li] = lse;
       }
-    } else {
-      *abort = 1;
     }
+    if (!ok) *abort = 1;
   }
 
   tc_fence_before_sync();
@@ -522,26 +680,48 @@ static unsigned int next_epoch() {
   return e;
 }
 
+struct DeviceInfo {
+  std::once_flag once;
+  int sm_count = 0;
+  cudaError_t attr_err[2] = {cudaSuccess, cudaSuccess};
+  int regs[2] = {0, 0};
+};
+
+static DeviceInfo g_devices[64];
+
 template <int D>
 static int launch(const void *q, const void *k, const void *v, const Params &p, int64_t tokens,
-                  int64_t grid, cudaStream_t stream) {
+                  cudaStream_t stream) {
   using C = KernelCfg<D>;
   CUtensorMap tq, tk, tv;
   if (!encode_tokens_heads_dim(&tq, q, tokens, p.Hq, D) ||
       !encode_tokens_heads_dim(&tk, k, tokens, p.Hkv, D) ||
       !encode_tokens_heads_dim(&tv, v, tokens, p.Hkv, D))
     return MK_ERR_CUDA;
-  static std::once_flag attr_once[64];
-  static cudaError_t attr_err[64];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return MK_ERR_CUDA;
-  std::call_once(attr_once[dev], [&] {
-    attr_err[dev] = cudaFuncSetAttribute(fmha_fwd_kernel<D>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         C::kSmemBytes);
+  DeviceInfo &di = g_devices[dev];
+  std::call_once(di.once, [&] {
+    if (cudaDeviceGetAttribute(&di.sm_count, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      di.sm_count = 0;
+    di.attr_err[0] = cudaFuncSetAttribute(fmha_fwd_kernel<64>,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          KernelCfg<64>::kSmemBytes);
+    di.attr_err[1] = cudaFuncSetAttribute(fmha_fwd_kernel<128>,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          KernelCfg<128>::kSmemBytes);
+    cudaFuncAttributes fa;
+    if (cudaFuncGetAttributes(&fa, fmha_fwd_kernel<64>) == cudaSuccess) di.regs[0] = fa.numRegs;
+    if (cudaFuncGetAttributes(&fa, fmha_fwd_kernel<128>) == cudaSuccess) di.regs[1] = fa.numRegs;
   });
-  if (attr_err[dev] != cudaSuccess) return MK_ERR_CUDA;
-  fmha_fwd_kernel<D><<<(unsigned)grid, kThreads, C::kSmemBytes, stream>>>(tq, tk, tv, p);
+  const int vi = D == 128 ? 1 : 0;
+  if (di.sm_count <= 0 || di.attr_err[vi] != cudaSuccess) return MK_ERR_CUDA;
+  // The warpgroup register split assumes the block launches with exactly
+  // kLaunchRegs registers per thread; anything else could leave a
+  // setmaxnreg.inc waiting forever, so refuse to launch.
+  if (di.regs[vi] != kLaunchRegs) return MK_ERR_CUDA;
+  const int grid = p.n_units < di.sm_count ? p.n_units : di.sm_count;
+  fmha_fwd_kernel<D><<<grid, kThreads, C::kSmemBytes, stream>>>(tq, tk, tv, p);
   return cudaGetLastError() == cudaSuccess ? MK_OK : MK_ERR_CUDA;
 }
 
@@ -566,11 +746,13 @@ int mk_attn_fwd(const void *q, const void *k, const void *v, void *o, float *lse
   const bool varlen = cu_seqlens != nullptr;
   const int64_t tokens = varlen ? (int64_t)S : (int64_t)B * S;
   if (tokens > INT32_MAX) return MK_ERR_INVALID_ARG;
-  // Work tiles: fixed length B * Hq * ceil(S/128); varlen at most
-  // Hq * (T + 127 B) / 128 (each sequence wastes under one tile).
-  const int64_t n_qtiles = varlen ? ((int64_t)S + 127LL * B) / kTile : ((int64_t)S + kTile - 1) / kTile;
-  const int64_t grid = varlen ? n_qtiles * Hq : n_qtiles * B * Hq;
-  if (grid > INT32_MAX || (int64_t)Hq * tokens > INT32_MAX * 64LL) return MK_ERR_INVALID_ARG;
+  // Work units (pairs of 128-row query tiles): fixed length B * Hq *
+  // ceil(ceil(S/128)/2); varlen at most Hq * (T + 255 B) / 256, since a
+  // sequence of L tokens has ceil(ceil(L/128)/2) <= L/256 + 1 pairs.
+  const int64_t n_pairs = (((int64_t)S + kTile - 1) / kTile + 1) / 2;
+  const int64_t n_units = varlen ? (int64_t)Hq * (((int64_t)S + 255LL * B) / 256)
+                                 : n_pairs * B * Hq;
+  if (n_units > INT32_MAX || n_units < 1) return MK_ERR_INVALID_ARG;
 
   Params p;
   p.o = reinterpret_cast<uint16_t *>(o);
@@ -583,12 +765,12 @@ int mk_attn_fwd(const void *q, const void *k, const void *v, void *o, float *lse
   p.group = Hq / Hkv;
   p.causal = causal != 0;
   p.varlen = varlen;
-  p.n_qtiles = (int)n_qtiles;
+  p.n_pairs = (int)n_pairs;
+  p.n_units = (int)n_units;
   p.scale_log2 = scale * 1.4426950408889634f;
   p.epoch = next_epoch();
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  return D == 128 ? launch<128>(q, k, v, p, tokens, grid, st)
-                  : launch<64>(q, k, v, p, tokens, grid, st);
+  return D == 128 ? launch<128>(q, k, v, p, tokens, st) : launch<64>(q, k, v, p, tokens, st);
 }
 
 const char *mk_attn_error_string(int status) {
@@ -616,6 +798,6 @@ int mk_attn_check_status(void *stream) {
   return MK_OK;
 }
 
-int mk_attn_version(void) { return 100; }
+int mk_attn_version(void) { return 200; }
 
 }  // extern "C"
