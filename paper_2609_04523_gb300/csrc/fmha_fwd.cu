@@ -83,8 +83,7 @@ struct KernelCfg {
 
 struct SharedCtl {
   uint64_t bar_q_full[2], bar_q_empty[2];
-  uint64_t bar_k_full[4], bar_k_empty[4];
-  uint64_t bar_v_full[4], bar_v_empty[4];
+  uint64_t bar_kv_full[4], bar_kv_empty[4];  // K/V slots
   uint64_t bar_s_full[2], bar_p_full[2];
   uint64_t bar_o_final[2];
   uint64_t bar_mma_drained;
@@ -226,10 +225,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&ctl->bar_o_final[x], 1);
     }
     for (int s = 0; s < NS; ++s) {
-      mbar_init(&ctl->bar_k_full[s], 1);
-      mbar_init(&ctl->bar_k_empty[s], 1);
-      mbar_init(&ctl->bar_v_full[s], 1);
-      mbar_init(&ctl->bar_v_empty[s], 1);
+      mbar_init(&ctl->bar_kv_full[s], 1);
+      mbar_init(&ctl->bar_kv_empty[s], 1);
     }
     mbar_init(&ctl->bar_mma_drained, 1);
     ctl->abort = 0;
@@ -251,21 +248,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     setmaxnreg_dec<kRegsCtl>();
     // The producer and MMA warps run their loops and waits with all 32 lanes
     // converged; one lane chosen by elect.sync issues each TMA / tcgen05
-    // instruction.  Keeping the warp converged lets the unit bookkeeping and
-    // the matrix descriptors live in warp-uniform registers, so consecutive
-    // tcgen05.mma issue back to back.
+    // instruction, so the bookkeeping and descriptors stay warp-uniform.
+    //
+    // K/V slots: iteration j of a unit (j = 0..n, n = key blocks of the unit)
+    // uses slot (global iteration) % NS, which holds K_j (for S(j) = Q K_j^T,
+    // j < n) and V_{j-1} (for O += P(j-1) V_{j-1}, j >= 1).  One full and one
+    // empty barrier per slot: one wait and one commit per iteration.
     if (warp == kLoadWarp) {
       // ---------------------------------------------------------- producer
-      uint64_t pol_q = 0, pol_kv = 0;
       if (elect_one()) {
         tma_prefetch_desc(&tm_q);
         tma_prefetch_desc(&tm_k);
         tma_prefetch_desc(&tm_v);
       }
-      pol_q = l2_policy_evict_first();
-      pol_kv = l2_policy_evict_last();
-      uint32_t q_iter = 0, kv_iter = 0;
-      uint32_t k_issued = 0, v_issued = 0;  // loads issued, for the drain below
+      const uint64_t pol_q = l2_policy_evict_first();
+      const uint64_t pol_kv = l2_policy_evict_last();
+      uint32_t q_iter = 0, it = 0;
       bool ok = true;
       for (int u = blockIdx.x; ok && u < p.n_units; u += gridDim.x) {
         const Unit w = map_unit(p, cu_smem, u);
@@ -273,7 +271,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int hkv = w.hq / p.group;
         const int n_blk = max(tile_blocks(p, w, 0), tile_blocks(p, w, 1));
         for (int x = 0; x < 2; ++x) {
-          ok = __all_sync(0xffffffffu, mbar_wait(&ctl->bar_q_empty[x], (q_iter & 1) ^ 1, abort));
+          ok = mbar_wait_all(&ctl->bar_q_empty[x], (q_iter & 1) ^ 1, abort);
           if (!ok) break;
           if (elect_one()) {
             mbar_arrive_expect_tx(&ctl->bar_q_full[x], C::kTileBytes);
@@ -287,43 +285,38 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (!ok) break;
         ++q_iter;
-        for (int j = 0; j < n_blk; ++j, ++kv_iter) {
-          const int s = kv_iter % NS;
-          const uint32_t ph = (kv_iter / NS) & 1;
-          ok = __all_sync(0xffffffffu, mbar_wait(&ctl->bar_k_empty[s], ph ^ 1, abort));
+        for (int j = 0; j <= n_blk; ++j) {
+          const int s = it % NS;
+          ok = mbar_wait_all(&ctl->bar_kv_empty[s], ((it / NS) & 1) ^ 1, abort);
           if (!ok) break;
           if (elect_one()) {
-            mbar_arrive_expect_tx(&ctl->bar_k_full[s], C::kTileBytes);
+            const uint32_t bytes = (j < n_blk ? C::kTileBytes : 0) + (j > 0 ? C::kTileBytes : 0);
+            mbar_arrive_expect_tx(&ctl->bar_kv_full[s], bytes);
+            if (j < n_blk) {
 #pragma unroll
-            for (int h = 0; h < C::kHalves; ++h)
-              tma_load_3d(smem + C::kOffK + s * C::kTileBytes + h * kBoxBytes, &tm_k,
-                          &ctl->bar_k_full[s], h * kBoxCols, hkv, w.seq_start + j * kTile,
-                          pol_kv);
+              for (int h = 0; h < C::kHalves; ++h)
+                tma_load_3d(smem + C::kOffK + s * C::kTileBytes + h * kBoxBytes, &tm_k,
+                            &ctl->bar_kv_full[s], h * kBoxCols, hkv, w.seq_start + j * kTile,
+                            pol_kv);
+            }
+            if (j > 0) {
+#pragma unroll
+              for (int h = 0; h < C::kHalves; ++h)
+                tma_load_3d(smem + C::kOffV + s * C::kTileBytes + h * kBoxBytes, &tm_v,
+                            &ctl->bar_kv_full[s], h * kBoxCols, hkv,
+                            w.seq_start + (j - 1) * kTile, pol_kv);
+            }
           }
           __syncwarp();
-          k_issued = kv_iter + 1;
-          ok = __all_sync(0xffffffffu, mbar_wait(&ctl->bar_v_empty[s], ph ^ 1, abort));
-          if (!ok) break;
-          if (elect_one()) {
-            mbar_arrive_expect_tx(&ctl->bar_v_full[s], C::kTileBytes);
-#pragma unroll
-            for (int h = 0; h < C::kHalves; ++h)
-              tma_load_3d(smem + C::kOffV + s * C::kTileBytes + h * kBoxBytes, &tm_v,
-                          &ctl->bar_v_full[s], h * kBoxCols, hkv, w.seq_start + j * kTile,
-                          pol_kv);
-          }
-          __syncwarp();
-          v_issued = kv_iter + 1;
+          ++it;
         }
       }
       // Teardown: every load issued must land before the CTA exits.  For each
-      // stage the last issued phase is waited for (earlier phases precede it).
+      // slot the last issued phase is waited for (earlier phases precede it).
       if (q_iter > 0)
         for (int x = 0; x < 2; ++x) drain_wait(&ctl->bar_q_full[x], (q_iter - 1) & 1);
-      for (uint32_t n = (k_issued > (uint32_t)NS ? k_issued - NS : 0); n < k_issued; ++n)
-        drain_wait(&ctl->bar_k_full[n % NS], (n / NS) & 1);
-      for (uint32_t n = (v_issued > (uint32_t)NS ? v_issued - NS : 0); n < v_issued; ++n)
-        drain_wait(&ctl->bar_v_full[n % NS], (n / NS) & 1);
+      for (uint32_t n = (it > (uint32_t)NS ? it - NS : 0); n < it; ++n)
+        drain_wait(&ctl->bar_kv_full[n % NS], (n / NS) & 1);
     } else if (warp == kMmaWarp) {
       // ---------------------------------------------------------- MMA issuer
       constexpr uint32_t idesc_qk = idesc_bf16_f32(kTile, kTile, false, false);
@@ -339,11 +332,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t dk0 = sdesc_sw128(sK, 16, 1024);
       const uint64_t dv0 = sdesc_sw128(sV, kVLbo, 1024);
       constexpr uint64_t kTileStep = C::kTileBytes >> 4;
-      uint32_t q_iter = 0, kv_iter = 0;
+      uint32_t q_iter = 0, it = 0;
       uint32_t p_cnt[2] = {0, 0};
       bool ok = true;
 
-      // S_X = Q_X K^T for the K tile in stage s (elected lane only).
+      // S_X = Q_X K^T for the K tile in slot s (elected lane only).
       auto issue_s = [&](int x, int s) {
         const uint64_t a0 = dq0 + x * kTileStep;
         const uint64_t b0 = dk0 + s * kTileStep;
@@ -355,7 +348,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         umma_commit(&ctl->bar_s_full[x]);
       };
-      // O_X (+)= P_X V for the V tile in stage s (elected lane only).
+      // O_X (+)= P_X V for the V tile in slot s (elected lane only).
       auto issue_pv = [&](int x, int s, bool first) {
         const uint64_t b0 = dv0 + s * kTileStep;
         const uint32_t d_tmem = tmem + kColO + x * D;
@@ -369,68 +362,47 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int u = blockIdx.x; ok && u < p.n_units; u += gridDim.x) {
         const Unit w = map_unit(p, cu_smem, u);
         if (!w.valid) continue;
-        const int n0 = tile_blocks(p, w, 0);
-        const int n1 = tile_blocks(p, w, 1);
-        const int n_blk = max(n0, n1);
+        const int nx[2] = {tile_blocks(p, w, 0), tile_blocks(p, w, 1)};
+        const int n_blk = max(nx[0], nx[1]);
         for (int x = 0; x < 2 && ok; ++x)
-          ok = __all_sync(0xffffffffu, mbar_wait(&ctl->bar_q_full[x], q_iter & 1, abort));
-        // j = 0: S_A(0), S_B(0)
-        int s_cur = kv_iter % NS;
-        if (ok)
-          ok = __all_sync(0xffffffffu,
-                          mbar_wait(&ctl->bar_k_full[s_cur], (kv_iter / NS) & 1, abort));
-        if (ok) {
-          tc_fence_after_sync();
-          if (elect_one()) {
-            if (n0 > 0) issue_s(0, s_cur);
-            if (n0 <= 1) umma_commit(&ctl->bar_q_empty[0]);  // Q_A no longer read
-            if (n1 > 0) issue_s(1, s_cur);
-            if (n1 <= 1) umma_commit(&ctl->bar_q_empty[1]);
-            umma_commit(&ctl->bar_k_empty[s_cur]);
-          }
-          __syncwarp();
-        }
-        for (int j = 1; ok && j <= n_blk; ++j) {
-          const uint32_t it_prev = kv_iter + j - 1;
-          const int s_prev = it_prev % NS;
-          const bool has_next = j < n_blk;
-          const uint32_t it_cur = kv_iter + j;
-          s_cur = it_cur % NS;
-          ok = __all_sync(0xffffffffu,
-                          mbar_wait(&ctl->bar_v_full[s_prev], (it_prev / NS) & 1, abort));
-          if (ok && has_next)
-            ok = __all_sync(0xffffffffu,
-                            mbar_wait(&ctl->bar_k_full[s_cur], (it_cur / NS) & 1, abort));
+          ok = mbar_wait_all(&ctl->bar_q_full[x], q_iter & 1, abort);
+        // Issue order per iteration j (ping-pong): wait slot, then for A and B
+        // in turn: wait P_X(j-1), O_X += P_X(j-1) V_{j-1}, S_X(j) = Q_X K_j^T.
+        // S_X(j) overwrites P_X(j-1) in TMEM, so it follows the P_X V that
+        // reads it.  The waits fall where earlier MMAs are still queued.
+        for (int j = 0; ok && j <= n_blk; ++j) {
+          const int s = it % NS;
+          ok = mbar_wait_all(&ctl->bar_kv_full[s], (it / NS) & 1, abort);
 #pragma unroll
           for (int x = 0; x < 2; ++x) {
-            const int nx = x == 0 ? n0 : n1;
-            if (ok && j - 1 < nx) {
-              ok = __all_sync(0xffffffffu,
-                              mbar_wait(&ctl->bar_p_full[x], p_cnt[x] & 1, abort));
-              ++p_cnt[x];
-            }
             if (!ok) break;
+            const bool do_pv = j > 0 && j - 1 < nx[x];
+            const bool do_s = j < nx[x];
+            if (do_pv) {
+              ok = mbar_wait_all(&ctl->bar_p_full[x], p_cnt[x] & 1, abort);
+              ++p_cnt[x];
+              if (!ok) break;
+            }
             tc_fence_after_sync();
             if (elect_one()) {
-              if (j - 1 < nx) {
-                issue_pv(x, s_prev, j == 1);
-                if (j - 1 == nx - 1) umma_commit(&ctl->bar_o_final[x]);
+              if (do_pv) {
+                issue_pv(x, s, j == 1);
+                if (j == nx[x]) umma_commit(&ctl->bar_o_final[x]);
               }
-              if (has_next && j < nx) {
-                issue_s(x, s_cur);
-                if (j == nx - 1) umma_commit(&ctl->bar_q_empty[x]);
+              if (do_s) {
+                issue_s(x, s);
+                if (j == nx[x] - 1) umma_commit(&ctl->bar_q_empty[x]);  // Q_X no longer read
+              } else if (j == 0) {
+                umma_commit(&ctl->bar_q_empty[x]);  // tile X lies past the sequence end
               }
             }
             __syncwarp();
           }
           if (!ok) break;
-          if (elect_one()) {
-            umma_commit(&ctl->bar_v_empty[s_prev]);
-            if (has_next) umma_commit(&ctl->bar_k_empty[s_cur]);
-          }
+          if (elect_one()) umma_commit(&ctl->bar_kv_empty[s]);
           __syncwarp();
+          ++it;
         }
-        kv_iter += n_blk;
         ++q_iter;
       }
       // Teardown: all MMAs issued by this warp complete before TMEM is freed.
@@ -466,12 +438,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       float l_run = 0.f;        // running row sum relative to m_run
 
       for (int j = 0; j < n_blk; ++j) {
-        ok = mbar_wait(&ctl->bar_s_full[X], s_cnt & 1, abort);
+        ok = mbar_wait_all(&ctl->bar_s_full[X], s_cnt & 1, abort);
         ++s_cnt;
-        if (!__all_sync(0xffffffffu, ok)) {
-          ok = false;
-          break;
-        }
+        if (!ok) break;
         tc_fence_after_sync();
         const bool needs_mask = (j * kTile + kTile > w.len) || (p.causal && j == qt);
         const int lim = key_limit - j * kTile;
@@ -555,7 +524,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_st_wait();
           load_scores(s);
         }
-        // p = 2^(s * c2 - m), one packed FMA per pair of keys.
+        // p = 2^(s * c2 - m): one FMA and one MUFU ex2 per key.
         const float neg_m = (m_run == -INFINITY) ? 0.f : -m_run;
         float sum0 = 0.f, sum1 = 0.f, sum2 = 0.f, sum3 = 0.f;
         uint32_t pk[2][32];
@@ -588,12 +557,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
 
       // ---------------------------------------------------------- epilogue
-      ok = mbar_wait(&ctl->bar_o_final[X], o_cnt & 1, abort);
+      ok = mbar_wait_all(&ctl->bar_o_final[X], o_cnt & 1, abort);
       ++o_cnt;
-      if (!__all_sync(0xffffffffu, ok)) {
-        ok = false;
-        break;
-      }
+      if (!ok) break;
       tc_fence_after_sync();
       const float inv_l = 1.f / l_run;
       const int64_t tok = (int64_t)w.seq_start + qpos;

@@ -115,6 +115,16 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volati
   }
 }
 
+// Warp-wide wait, called by all 32 lanes of a converged warp: one poll and
+// one vote on the fast path (the phase has already completed), the bounded
+// spin otherwise.  Returns the same value in every lane.
+__device__ __forceinline__ bool mbar_wait_all(uint64_t *bar, uint32_t parity,
+                                              volatile int *abort) {
+  const uint32_t a = smem_addr(bar);
+  if (__all_sync(0xffffffffu, mbar_try_wait(a, parity))) return true;
+  return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort));
+}
+
 // --------------------------------------------------------------------- TMA
 
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap *map) {
