@@ -184,6 +184,15 @@ __device__ __forceinline__ int tile_blocks(const Params &p, const Unit &w, int X
   return p.causal ? min(qt + 1, n_kb) : n_kb;
 }
 
+// Unit processed by this CTA in round k.  Units are numbered heaviest first
+// (fixed-length causal); rounds alternate direction over the CTAs (CTA c takes
+// unit kG + c in even rounds and kG + G - 1 - c in odd ones), which balances
+// the per-CTA sums of decreasing unit costs far better than plain round-robin.
+__device__ __forceinline__ int unit_of_round(int k) {
+  const int G = gridDim.x, c = blockIdx.x;
+  return (k & 1) ? (k + 1) * G - 1 - c : k * G + c;
+}
+
 // Bounded wait that ignores the abort flag: used only at teardown to let
 // operations already in flight land before the CTA releases its resources.
 __device__ __forceinline__ void drain_wait(uint64_t *bar, uint32_t parity) {
@@ -265,7 +274,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t pol_kv = l2_policy_evict_last();
       uint32_t q_iter = 0, it = 0;
       bool ok = true;
-      for (int u = blockIdx.x; ok && u < p.n_units; u += gridDim.x) {
+      for (int k = 0; ok && k * (int)gridDim.x < p.n_units; ++k) {
+        const int u = unit_of_round(k);
+        if (u >= p.n_units) continue;
         const Unit w = map_unit(p, cu_smem, u);
         if (!w.valid) continue;
         const int hkv = w.hq / p.group;
@@ -359,7 +370,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                   (!first || kk > 0) ? 1u : 0u);
       };
 
-      for (int u = blockIdx.x; ok && u < p.n_units; u += gridDim.x) {
+      for (int k = 0; ok && k * (int)gridDim.x < p.n_units; ++k) {
+        const int u = unit_of_round(k);
+        if (u >= p.n_units) continue;
         const Unit w = map_unit(p, cu_smem, u);
         if (!w.valid) continue;
         const int nx[2] = {tile_blocks(p, w, 0), tile_blocks(p, w, 1)};
@@ -425,7 +438,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t s_cnt = 0, o_cnt = 0;
     bool ok = true;
 
-    for (int u = blockIdx.x; ok && u < p.n_units; u += gridDim.x) {
+    for (int k = 0; ok && k * (int)gridDim.x < p.n_units; ++k) {
+        const int u = unit_of_round(k);
+        if (u >= p.n_units) continue;
       const Unit w = map_unit(p, cu_smem, u);
       if (!w.valid) continue;
       const int n_blk = tile_blocks(p, w, X);
