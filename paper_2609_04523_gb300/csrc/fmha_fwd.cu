@@ -434,6 +434,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t t_o = t_row + kColO + X * D;
     const float c2 = p.scale_log2;
     const bool neg_scale = c2 < 0.f;
+    const bool zero_scale = c2 == 0.f;
     const float mask_val = neg_scale ? INFINITY : -INFINITY;
     uint32_t s_cnt = 0, o_cnt = 0;
     bool ok = true;
@@ -550,7 +551,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           ffma2_bcast(a2, a3, s[c + 2], s[c + 3], c2, neg_m);
           float p0 = ex2_approx(a0), p1 = ex2_approx(a1);
           float p2 = ex2_approx(a2), p3 = ex2_approx(a3);
-          if (needs_mask) {
+          // A hidden key's score is +-inf with the sign that makes s * c2 = -inf,
+          // so p = 0 already; only c2 = 0 (0 * inf = NaN) needs the select.
+          if (needs_mask && zero_scale) {
             p0 = (c < lim) ? p0 : 0.f;
             p1 = (c + 1 < lim) ? p1 : 0.f;
             p2 = (c + 2 < lim) ? p2 : 0.f;
