@@ -94,6 +94,21 @@ def test_gqa_groups(D, G, B):
     check_fixed(B=B, Hq=8, Hkv=8 // G, S=300, D=D, causal=True, seed=100 + G * 10 + B + D)
 
 
+@pytest.mark.parametrize("causal", [True, False])
+def test_gqa_odd_group(causal):
+    """G = 3: units pair consecutive row tiles of one head (no head pairs)."""
+    check_fixed(B=2, Hq=6, Hkv=2, S=700, D=128, causal=causal, seed=150 + int(causal))
+
+
+@pytest.mark.parametrize("causal", [True, False])
+def test_varlen_gqa_odd_group(causal):
+    lens = [300, 129, 1, 640]
+    q, k, v, cu = W.make_qkv(0, 6, 2, 0, 64, seed=160, lengths=lens)
+    o, lse = gpu_attn(q, k, v, causal, 0.125, cu)
+    o_ref, lse_ref = oracle.attn_fwd(q, k, v, causal, 0.125, cu_seqlens=cu.numpy())
+    assert_close(o, lse, o_ref, lse_ref, "varlen G=3")
+
+
 @pytest.mark.parametrize("D", [64, 128])
 def test_long_noncausal(D):
     check_fixed(B=1, Hq=2, Hkv=1, S=1000, D=D, causal=False, seed=200 + D)
