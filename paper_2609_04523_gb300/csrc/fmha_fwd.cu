@@ -434,8 +434,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t t_o = t_row + kColO + X * D;
     const float c2 = p.scale_log2;
     const bool neg_scale = c2 < 0.f;
-    const bool zero_scale = c2 == 0.f;
-    const float mask_val = neg_scale ? INFINITY : -INFINITY;
+    const float c2a = fmaxf(fabsf(c2), 1.17549435e-38f);  // |c2|, at least FLT_MIN
     uint32_t s_cnt = 0, o_cnt = 0;
     bool ok = true;
 
@@ -460,9 +459,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after_sync();
         const bool needs_mask = (j * kTile + kTile > w.len) || (p.causal && j == qt);
         const int lim = key_limit - j * kTile;
-        // s = raw S_X(j) row.  Hidden keys take the value that loses the
-        // max (min when scale < 0), and get p = 0 after the exponential, so the
-        // mask holds for every sign of the scale, zero included.
+        // s = S_X(j) row in the form the exponential takes: negated when the
+        // scale is negative (t = s * c2 = (-s) * |c2|), hidden keys at -inf.
+        // With c2a = max(|c2|, FLT_MIN) > 0 a hidden key gives p = 2^-inf = 0
+        // and the row max is c2a * max(s).  (For c2 = 0, every visible
+        // s * FLT_MIN is at most a denormal, which ex2.approx.ftz reads as 0:
+        // p = 1, exactly as for a zero scale.)  The exponential loop below is
+        // branch-free: a branch inside it would stop the scheduler from
+        // overlapping the MUFU latencies of consecutive keys.
         auto load_scores = [&](float (&s)[kTile]) {
           uint32_t raw[4][32];
 #pragma unroll
@@ -474,44 +478,28 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int e = 0; e < 32; ++e) s[c * 32 + e] = __uint_as_float(raw[c][e]);
           }
+          if (neg_scale) {
+#pragma unroll
+            for (int c = 0; c < kTile; ++c) s[c] = -s[c];
+          }
           if (needs_mask) {
 #pragma unroll
-            for (int c = 0; c < kTile; ++c) s[c] = (c < lim) ? s[c] : mask_val;
+            for (int c = 0; c < kTile; ++c) s[c] = (c < lim) ? s[c] : -INFINITY;
           }
         };
         float s[kTile];
         load_scores(s);
-        // Row max of t = s * c2 (base-2 units) = c2 * (max s), or c2 * (min s)
-        // when c2 < 0.
-        float mx0, mx1, mx2, mx3;
-        if (!neg_scale) {
-          mx0 = fmaxf(s[0], s[1]);
-          mx1 = fmaxf(s[2], s[3]);
-          mx2 = fmaxf(s[4], s[5]);
-          mx3 = fmaxf(s[6], s[7]);
+        float mx0 = fmaxf(s[0], s[1]), mx1 = fmaxf(s[2], s[3]);
+        float mx2 = fmaxf(s[4], s[5]), mx3 = fmaxf(s[6], s[7]);
 #pragma unroll
-          for (int c = 8; c < kTile; c += 8) {
-            mx0 = fmax3(mx0, s[c], s[c + 1]);
-            mx1 = fmax3(mx1, s[c + 2], s[c + 3]);
-            mx2 = fmax3(mx2, s[c + 4], s[c + 5]);
-            mx3 = fmax3(mx3, s[c + 6], s[c + 7]);
-          }
-          mx0 = fmaxf(fmax3(mx0, mx1, mx2), mx3);
-        } else {
-          mx0 = fminf(s[0], s[1]);
-          mx1 = fminf(s[2], s[3]);
-          mx2 = fminf(s[4], s[5]);
-          mx3 = fminf(s[6], s[7]);
-#pragma unroll
-          for (int c = 8; c < kTile; c += 8) {
-            mx0 = fmin3(mx0, s[c], s[c + 1]);
-            mx1 = fmin3(mx1, s[c + 2], s[c + 3]);
-            mx2 = fmin3(mx2, s[c + 4], s[c + 5]);
-            mx3 = fmin3(mx3, s[c + 6], s[c + 7]);
-          }
-          mx0 = fminf(fmin3(mx0, mx1, mx2), mx3);
+        for (int c = 8; c < kTile; c += 8) {
+          mx0 = fmax3(mx0, s[c], s[c + 1]);
+          mx1 = fmax3(mx1, s[c + 2], s[c + 3]);
+          mx2 = fmax3(mx2, s[c + 4], s[c + 5]);
+          mx3 = fmax3(mx3, s[c + 6], s[c + 7]);
         }
-        const float m_new = fmaxf(m_run, mx0 * c2);  // fmaxf drops a NaN (0 * inf)
+        mx0 = fmaxf(fmax3(mx0, mx1, mx2), mx3);
+        const float m_new = fmaxf(m_run, mx0 * c2a);
         // Lazy rescaling: keep the old reference max unless the new one exceeds
         // it by more than the threshold.  Exact either way, because O and l
         // always share the same reference max.
@@ -540,25 +528,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_st_wait();
           load_scores(s);
         }
-        // p = 2^(s * c2 - m): one FMA and one MUFU ex2 per key.
+        // p = 2^(s * c2a - m): one FMA and one MUFU ex2 per key.
         const float neg_m = (m_run == -INFINITY) ? 0.f : -m_run;
         float sum0 = 0.f, sum1 = 0.f, sum2 = 0.f, sum3 = 0.f;
         uint32_t pk[2][32];
 #pragma unroll
         for (int c = 0; c < kTile; c += 4) {
           float a0, a1, a2, a3;
-          ffma2_bcast(a0, a1, s[c], s[c + 1], c2, neg_m);
-          ffma2_bcast(a2, a3, s[c + 2], s[c + 3], c2, neg_m);
-          float p0 = ex2_approx(a0), p1 = ex2_approx(a1);
-          float p2 = ex2_approx(a2), p3 = ex2_approx(a3);
-          // A hidden key's score is +-inf with the sign that makes s * c2 = -inf,
-          // so p = 0 already; only c2 = 0 (0 * inf = NaN) needs the select.
-          if (needs_mask && zero_scale) {
-            p0 = (c < lim) ? p0 : 0.f;
-            p1 = (c + 1 < lim) ? p1 : 0.f;
-            p2 = (c + 2 < lim) ? p2 : 0.f;
-            p3 = (c + 3 < lim) ? p3 : 0.f;
-          }
+          ffma2_bcast(a0, a1, s[c], s[c + 1], c2a, neg_m);
+          ffma2_bcast(a2, a3, s[c + 2], s[c + 3], c2a, neg_m);
+          const float p0 = ex2_approx(a0), p1 = ex2_approx(a1);
+          const float p2 = ex2_approx(a2), p3 = ex2_approx(a3);
           fadd2_acc(sum0, sum1, p0, p1);
           fadd2_acc(sum2, sum3, p2, p3);
           pk[c / 64][(c % 64) / 2] = pack_bf16x2(p0, p1);
