@@ -294,6 +294,15 @@ __device__ __forceinline__ void reg_fence(uint32_t (&r)[32]) {
                       "+r"(r[i + 4]), "+r"(r[i + 5]), "+r"(r[i + 6]), "+r"(r[i + 7]));
 }
 
+// 256-bit global store (sm_100+); `ptr` must be 32-byte aligned.
+__device__ __forceinline__ void st_global_v8(void *ptr, uint32_t a0, uint32_t a1, uint32_t a2,
+                                             uint32_t a3, uint32_t a4, uint32_t a5, uint32_t a6,
+                                             uint32_t a7) {
+  asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(ptr), "r"(a0),
+               "r"(a1), "r"(a2), "r"(a3), "r"(a4), "r"(a5), "r"(a6), "r"(a7)
+               : "memory");
+}
+
 // ------------------------------------------------------------------ scalars
 
 // 2^x on the MUFU unit (approximate, flush-to-zero; 2^-inf = +0).

@@ -255,6 +255,24 @@ def test_guard_regions_untouched():
     assert_close(o.cpu(), lse.cpu(), o_ref, lse_ref, "guarded")
 
 
+@pytest.mark.parametrize("offset_bytes", [16, 32])
+def test_output_pointer_alignment(offset_bytes):
+    """o at a 16-byte (not 32-byte) and at a 32-byte aligned address: the
+    epilogue switches between 16- and 32-byte stores; both must agree."""
+    dev = torch.device("cuda")
+    B, S, Hq, Hkv, D = 1, 260, 4, 2, 128
+    q, k, v, _ = W.make_qkv(B, Hq, Hkv, S, D, seed=505)
+    n_o = B * S * Hq * D
+    base = torch.zeros(n_o + 64, dtype=torch.bfloat16, device=dev)
+    assert base.data_ptr() % 256 == 0
+    o = base[offset_bytes // 2: offset_bytes // 2 + n_o].view(B, S, Hq, D)
+    lse = torch.empty((B, Hq, S), dtype=torch.float32, device=dev)
+    binding.attn_fwd(q.to(dev), k.to(dev), v.to(dev), True, 0.1, None, out=o, lse=lse)
+    assert binding.mk_attn_check_status(torch.cuda.current_stream().cuda_stream) == 0
+    o_ref, lse_ref = oracle.attn_fwd(q, k, v, True, 0.1)
+    assert_close(o.cpu(), lse.cpu(), o_ref, lse_ref, f"o offset {offset_bytes}")
+
+
 def test_rejected_call_leaves_outputs_untouched():
     dev = torch.device("cuda")
     q, k, v, _ = W.make_qkv(1, 4, 2, 64, 64, seed=504)
