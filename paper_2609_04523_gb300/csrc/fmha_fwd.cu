@@ -65,7 +65,6 @@ constexpr float kRescaleThreshold = 8.0f;  // log2 units: rescale O when m rises
 constexpr int kCuCache = 2048;        // cu_seqlens entries cached in shared memory
 
 __device__ int g_status = 0;               // MK_ERR_TIMEOUT once a wait ran out
-__device__ unsigned int g_abort_epoch = 0;  // launch epoch that timed out
 
 template <int D>
 struct KernelCfg {
@@ -103,7 +102,6 @@ struct Params {
   int n_units;              // fixed: exact; varlen: upper bound
   float scale_log2;         // scale * log2(e)
   int o_align32;            // o is 32-byte aligned: 256-bit stores in the epilogue
-  unsigned int epoch;
 };
 
 struct Unit {
@@ -208,8 +206,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const __grid_constant__ CUtensorMap tm_v, const Params p) {
   using C = KernelCfg<D>;
   constexpr int NS = C::kStages;
-
-  if (*reinterpret_cast<volatile unsigned int *>(&g_abort_epoch) == p.epoch) return;
 
   extern __shared__ uint8_t smem_raw[];
   // 1024-byte alignment for the 128-byte-swizzle atoms.
@@ -608,7 +604,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   if (threadIdx.x == 0 && ctl->abort) {
     atomicExch(&g_status, (int)MK_ERR_TIMEOUT);
-    atomicExch(&g_abort_epoch, p.epoch);
   }
 }
 
@@ -640,16 +635,6 @@ static bool encode_tokens_heads_dim(CUtensorMap *map, const void *base, uint64_t
   return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides,
              box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-static std::atomic<unsigned int> g_epoch_counter{0};
-
-static unsigned int next_epoch() {
-  unsigned int e;
-  do {
-    e = g_epoch_counter.fetch_add(1) + 1;
-  } while (e == 0);
-  return e;
 }
 
 struct DeviceInfo {
@@ -741,7 +726,6 @@ int mk_attn_fwd(const void *q, const void *k, const void *v, void *o, float *lse
   p.n_units = (int)n_units;
   p.scale_log2 = scale * 1.4426950408889634f;
   p.o_align32 = (reinterpret_cast<uintptr_t>(o) & 31u) == 0;
-  p.epoch = next_epoch();
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   return D == 128 ? launch<128>(q, k, v, p, tokens, st) : launch<64>(q, k, v, p, tokens, st);
 }
