@@ -228,7 +228,9 @@ def cpu_oracle_sample(inp, seconds: float, seed: int):
     o, lse = oracle.attn_rows(inp.q, inp.k, inp.v, c.causal, c.scale, rows, cu_seqlens=cu)
     dt = time.perf_counter() - t0
     fl = flops_of(rows)
-    desc = (f"{len(rows)} uniformly drawn rows (sequence, head, position) of the workload, "
+    what = ("all rows (sequence, head, position) of the workload" if n == total_rows else
+            "uniformly drawn rows (sequence, head, position) of the workload")
+    desc = (f"{len(rows)} {what}, "
             f"{fl / 1e9:.1f} GFLOP (exact visible pairs x 4D), {dt:.1f} s on {cores} threads")
     return fl / dt / 1e12, cores, desc, rows, o, lse
 
