@@ -149,6 +149,22 @@ def check_zero_scale(lib):
                 _close(lse[b, 1, i], math.log(n), 1e-14, "scale 0 lse")
 
 
+def check_negative_scale(lib):
+    """scale < 0: scale * q.k = |scale| * (-q).k, and negating a bf16 value is
+    exact, so the oracle at (q, -c) equals the oracle at (-q, c) exactly; the
+    explicit-P formulation agrees at the negative scale too."""
+    B, Hq, Hkv, S, D = 2, 4, 2, 19, 16
+    q, k, v, _ = W.make_qkv(B, Hq, Hkv, S, D, seed=131)
+    for causal in (False, True):
+        o, lse = _run(lib, q, k, v, causal, -0.4)
+        o2, lse2 = _run(lib, -q, k, v, causal, 0.4)
+        _close(o, o2, 0.0, f"negated scale vs negated q o (causal {causal})")
+        _close(lse, lse2, 0.0, f"negated scale vs negated q lse (causal {causal})")
+        ob, lseb = brute.attn_fwd(_bits(q), _bits(k), _bits(v), causal, -0.4)
+        _close(o, ob, TIGHT, f"negative scale brute o (causal {causal})")
+        _close(lse, lseb, TIGHT, f"negative scale brute lse (causal {causal})")
+
+
 def check_one_hot_values(lib):
     """v_j = e_j (S <= D): o_i is row i of P itself.  Its entries are >= 0,
     sum to 1, vanish on hidden keys, and follow exp(s_ij - lse_i)."""
@@ -297,6 +313,7 @@ ALL_CHECKS = [
     check_identical_keys,
     check_single_key,
     check_zero_scale,
+    check_negative_scale,
     check_one_hot_values,
     check_adversarial_rows,
     check_gqa_equals_repeated_mha,
