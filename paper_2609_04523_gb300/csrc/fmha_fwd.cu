@@ -25,6 +25,8 @@
 // MMA issue order per key block j (ping-pong):
 //   O_A += P_A(j-1) V_{j-1};  S_A(j) = Q_A K_j^T;  O_B += P_B(j-1) V_{j-1};  S_B(j) = Q_B K_j^T
 // so the softmax of one tile runs while the tensor pipe works on the other.
+// P_X is published in two halves of 64 keys, each on its own barrier: the
+// MMA warp issues P_X V over keys 0..63 while keys 64..127 are exponentiated.
 // Because S_X(j) is issued after P_X(j-1) V_{j-1}, every MMA that touches O_X
 // has completed when S_X(j) has: the softmax warps rescale O_X in TMEM (lazily,
 // only when the row max rises by more than kRescaleThreshold) with no extra wait.
@@ -83,7 +85,8 @@ struct KernelCfg {
 struct SharedCtl {
   uint64_t bar_q_full[2], bar_q_empty[2];
   uint64_t bar_kv_full[4], bar_kv_empty[4];  // K/V slots
-  uint64_t bar_s_full[2], bar_p_full[2];
+  uint64_t bar_s_full[2];
+  uint64_t bar_p_full[2][2];  // [tile][half]: P_X keys 0..63, then keys 64..127
   uint64_t bar_o_final[2];
   uint64_t bar_mma_drained;
   uint32_t tmem_base;
@@ -227,7 +230,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&ctl->bar_q_full[x], 1);
       mbar_init(&ctl->bar_q_empty[x], 1);
       mbar_init(&ctl->bar_s_full[x], 1);
-      mbar_init(&ctl->bar_p_full[x], kSoftmaxThreads);
+      mbar_init(&ctl->bar_p_full[x][0], kSoftmaxThreads);
+      mbar_init(&ctl->bar_p_full[x][1], kSoftmaxThreads);
       mbar_init(&ctl->bar_o_final[x], 1);
     }
     for (int s = 0; s < NS; ++s) {
@@ -356,15 +360,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         umma_commit(&ctl->bar_s_full[x]);
       };
-      // O_X (+)= P_X V for the V tile in slot s (elected lane only).
-      auto issue_pv = [&](int x, int s, bool first) {
+      // O_X (+)= P_X V over keys 64 * half .. 64 * half + 63 of the V tile in
+      // slot s (elected lane only).
+      auto issue_pv = [&](int x, int s, int half, bool first) {
         const uint64_t b0 = dv0 + s * kTileStep;
         const uint32_t d_tmem = tmem + kColO + x * D;
         const uint32_t a_tmem = tmem + kColS + x * 128;
 #pragma unroll
-        for (int kk = 0; kk < kTile / 16; ++kk)
+        for (int k4 = 0; k4 < kTile / 32; ++k4) {
+          const int kk = half * (kTile / 32) + k4;
           umma_ts(d_tmem, a_tmem + kk * 8, b0 + (uint64_t)(kk * 128), idesc_pv,
                   (!first || kk > 0) ? 1u : 0u);
+        }
       };
 
       for (int k = 0; ok && k * (int)gridDim.x < p.n_units; ++k) {
@@ -389,14 +396,21 @@ __global__ void __launch_bounds__(kThreads, 1)
             const bool do_pv = j > 0 && j - 1 < nx[x];
             const bool do_s = j < nx[x];
             if (do_pv) {
-              ok = mbar_wait_all(&ctl->bar_p_full[x], p_cnt[x] & 1, abort);
+              // P_X(j-1) arrives in two halves; the first half's MMAs run
+              // while the softmax computes the second.
+              ok = mbar_wait_all(&ctl->bar_p_full[x][0], p_cnt[x] & 1, abort);
+              if (!ok) break;
+              tc_fence_after_sync();
+              if (elect_one()) issue_pv(x, s, 0, j == 1);
+              __syncwarp();
+              ok = mbar_wait_all(&ctl->bar_p_full[x][1], p_cnt[x] & 1, abort);
               ++p_cnt[x];
               if (!ok) break;
             }
             tc_fence_after_sync();
             if (elect_one()) {
               if (do_pv) {
-                issue_pv(x, s, j == 1);
+                issue_pv(x, s, 1, false);
                 if (j == nx[x]) umma_commit(&ctl->bar_o_final[x]);
               }
               if (do_s) {
@@ -528,26 +542,31 @@ __global__ void __launch_bounds__(kThreads, 1)
         // p = 2^(s * c2a - m): one FMA and one MUFU ex2 per key.
         const float neg_m = (m_run == -INFINITY) ? 0.f : -m_run;
         float sum0 = 0.f, sum1 = 0.f, sum2 = 0.f, sum3 = 0.f;
-        uint32_t pk[2][32];
+        // P_X(j) (bf16, 64 columns) overwrites the first half of S_X(j), in
+        // two halves of 64 keys (32 columns), each announced on its own
+        // barrier so that the MMA warp starts O_X += P V on keys 0..63 while
+        // keys 64..127 are still being exponentiated.
 #pragma unroll
-        for (int c = 0; c < kTile; c += 4) {
-          float a0, a1, a2, a3;
-          ffma2_bcast(a0, a1, s[c], s[c + 1], c2a, neg_m);
-          ffma2_bcast(a2, a3, s[c + 2], s[c + 3], c2a, neg_m);
-          const float p0 = ex2_approx(a0), p1 = ex2_approx(a1);
-          const float p2 = ex2_approx(a2), p3 = ex2_approx(a3);
-          fadd2_acc(sum0, sum1, p0, p1);
-          fadd2_acc(sum2, sum3, p2, p3);
-          pk[c / 64][(c % 64) / 2] = pack_bf16x2(p0, p1);
-          pk[c / 64][(c % 64) / 2 + 1] = pack_bf16x2(p2, p3);
+        for (int half = 0; half < 2; ++half) {
+          uint32_t pk[32];
+#pragma unroll
+          for (int c = half * 64; c < half * 64 + 64; c += 4) {
+            float a0, a1, a2, a3;
+            ffma2_bcast(a0, a1, s[c], s[c + 1], c2a, neg_m);
+            ffma2_bcast(a2, a3, s[c + 2], s[c + 3], c2a, neg_m);
+            const float p0 = ex2_approx(a0), p1 = ex2_approx(a1);
+            const float p2 = ex2_approx(a2), p3 = ex2_approx(a3);
+            fadd2_acc(sum0, sum1, p0, p1);
+            fadd2_acc(sum2, sum3, p2, p3);
+            pk[(c % 64) / 2] = pack_bf16x2(p0, p1);
+            pk[(c % 64) / 2 + 1] = pack_bf16x2(p2, p3);
+          }
+          tmem_st_32x32b_x32(t_s + half * 32, pk);
+          tmem_st_wait();
+          tc_fence_before_sync();
+          mbar_arrive(&ctl->bar_p_full[X][half]);
         }
         l_run += (sum0 + sum1) + (sum2 + sum3);
-        // P_X(j) (bf16, 64 columns) overwrites the first half of S_X(j).
-        tmem_st_32x32b_x32(t_s, pk[0]);
-        tmem_st_32x32b_x32(t_s + 32, pk[1]);
-        tmem_st_wait();
-        tc_fence_before_sync();
-        mbar_arrive(&ctl->bar_p_full[X]);
       }
       if (!ok) break;
 
