@@ -154,6 +154,28 @@ def test_zero_scale_gives_prefix_means():
     assert np.max(np.abs(lse[0, 0].double().numpy() - np.log(n))) <= LSE_MAX_ABS
 
 
+@pytest.mark.parametrize("D", [64, 128])
+@pytest.mark.parametrize("causal", [True, False])
+def test_negative_scale(D, causal):
+    """softmax(c q k^T) with c < 0: the row max of c s comes from the row's
+    smallest score, and hidden keys must still get weight 0."""
+    check_fixed(B=2, Hq=4, Hkv=2, S=300, D=D, causal=causal, seed=410 + D + int(causal),
+                scale=-1.0 / math.sqrt(D))
+
+
+def test_negative_scale_with_rescales():
+    """A steep negative scale over 1000 keys: the running max rises by more
+    than the lazy-rescale threshold many times along each row."""
+    check_fixed(B=1, Hq=2, Hkv=1, S=1000, D=128, causal=False, seed=414, scale=-0.7)
+
+
+def test_negative_zero_scale():
+    q, k, v, _ = W.make_qkv(1, 2, 2, 200, 64, seed=412)
+    o, lse = gpu_attn(q, k, v, True, -0.0)
+    o_ref, lse_ref = oracle.attn_fwd(q, k, v, True, 0.0)
+    assert_close(o, lse, o_ref, lse_ref, "scale -0")
+
+
 def test_identical_keys():
     q, k, v, _ = W.make_qkv(1, 4, 1, 260, 64, seed=401)
     k = k[:, :1].expand_as(k).contiguous()
