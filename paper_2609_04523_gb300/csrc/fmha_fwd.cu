@@ -383,11 +383,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int n_blk = max(nx[0], nx[1]);
         for (int x = 0; x < 2 && ok; ++x)
           ok = mbar_wait_all(&ctl->bar_q_full[x], q_iter & 1, abort);
-        // Issue order per iteration j (ping-pong): wait slot, then for A and B
-        // in turn: wait P_X(j-1), O_X += P_X(j-1) V_{j-1}, S_X(j) = Q_X K_j^T.
-        // S_X(j) overwrites P_X(j-1) in TMEM, so it follows the P_X V that
-        // reads it.  The waits fall where earlier MMAs are still queued.
-        for (int j = 0; ok && j <= n_blk; ++j) {
+        const int n_min = min(nx[0], nx[1]);
+        // Generic iteration j: any mix of P V and S per tile (unit edges).
+        auto edge_iteration = [&](int j) {
           const int s = it % NS;
           ok = mbar_wait_all(&ctl->bar_kv_full[s], (it / NS) & 1, abort);
 #pragma unroll
@@ -396,8 +394,6 @@ __global__ void __launch_bounds__(kThreads, 1)
             const bool do_pv = j > 0 && j - 1 < nx[x];
             const bool do_s = j < nx[x];
             if (do_pv) {
-              // P_X(j-1) arrives in two halves; the first half's MMAs run
-              // while the softmax computes the second.
               ok = mbar_wait_all(&ctl->bar_p_full[x][0], p_cnt[x] & 1, abort);
               if (!ok) break;
               tc_fence_after_sync();
@@ -413,12 +409,41 @@ __global__ void __launch_bounds__(kThreads, 1)
                 issue_pv(x, s, 1, false);
                 if (j == nx[x]) umma_commit(&ctl->bar_o_final[x]);
               }
-              if (do_s) {
-                issue_s(x, s);
-                if (j == nx[x] - 1) umma_commit(&ctl->bar_q_empty[x]);  // Q_X no longer read
-              } else if (j == 0) {
-                umma_commit(&ctl->bar_q_empty[x]);  // tile X lies past the sequence end
-              }
+              if (do_s) issue_s(x, s);
+              if (j == nx[x] - 1 || (j == 0 && nx[x] == 0))
+                umma_commit(&ctl->bar_q_empty[x]);  // Q_X no longer read
+            }
+            __syncwarp();
+          }
+          if (!ok) return;
+          if (elect_one()) umma_commit(&ctl->bar_kv_empty[s]);
+          __syncwarp();
+          ++it;
+        };
+        // Iteration 0 (S only), then the steady iterations 1 .. n_min - 1 in
+        // which both tiles do P V and S (no per-tile conditions), then the
+        // iterations in which only the longer tile still works.
+        if (ok) edge_iteration(0);
+        for (int j = 1; ok && j < n_min; ++j) {
+          const int s = it % NS;
+          ok = mbar_wait_all(&ctl->bar_kv_full[s], (it / NS) & 1, abort);
+#pragma unroll
+          for (int x = 0; x < 2; ++x) {
+            if (!ok) break;
+            // P_X(j-1) arrives in two halves; the first half's MMAs run
+            // while the softmax computes the second.
+            ok = mbar_wait_all(&ctl->bar_p_full[x][0], p_cnt[x] & 1, abort);
+            if (!ok) break;
+            tc_fence_after_sync();
+            if (elect_one()) issue_pv(x, s, 0, j == 1);
+            __syncwarp();
+            ok = mbar_wait_all(&ctl->bar_p_full[x][1], p_cnt[x] & 1, abort);
+            ++p_cnt[x];
+            if (!ok) break;
+            tc_fence_after_sync();
+            if (elect_one()) {
+              issue_pv(x, s, 1, false);
+              issue_s(x, s);
             }
             __syncwarp();
           }
@@ -427,6 +452,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();
           ++it;
         }
+        if (ok && n_min >= 2) {
+          // The shorter tile's last S (j = n_min - 1) was issued in the loop above.
+          if (elect_one()) {
+#pragma unroll
+            for (int x = 0; x < 2; ++x)
+              if (nx[x] == n_min) umma_commit(&ctl->bar_q_empty[x]);
+          }
+          __syncwarp();
+        }
+        for (int j = max(n_min, 1); ok && j <= n_blk; ++j) edge_iteration(j);
         ++q_iter;
       }
       // Teardown: all MMAs issued by this warp complete before TMEM is freed.
