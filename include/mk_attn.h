@@ -84,6 +84,20 @@ MK_API int mk_attn_fwd(const void *q, const void *k, const void *v, void *o, flo
                        int B, int Hq, int Hkv, int S, int D, int causal, float scale,
                        const int32_t *cu_seqlens, void *stream);
 
+/*
+ * mk_attn_fwd_stall_test -- test support for the failure path only.  Same
+ * arguments, checks and return value as mk_attn_fwd, but every CTA leaves its
+ * first K/V pipeline slot unsignalled: the kernel's bounded wait on that slot
+ * runs out (about 2 s), all roles of the CTA unwind (in-flight copies and
+ * MMAs are drained, tensor memory is freed), o and lse are left incomplete,
+ * and the next mk_attn_check_status on the stream returns MK_ERR_TIMEOUT.
+ * No fault is raised; the CUDA context stays usable.  Never needed for
+ * computing attention.
+ */
+MK_API int mk_attn_fwd_stall_test(const void *q, const void *k, const void *v, void *o,
+                                  float *lse, int B, int Hq, int Hkv, int S, int D, int causal,
+                                  float scale, const int32_t *cu_seqlens, void *stream);
+
 /* Short static description of a status code.  Never NULL. */
 MK_API const char *mk_attn_error_string(int status);
 

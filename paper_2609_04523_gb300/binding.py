@@ -21,7 +21,8 @@ MK_ERR_CUDA = -4
 MK_ERR_TIMEOUT = -5
 
 # Symbols declared in include/mk_attn.h.
-EXPORTED = ("mk_attn_fwd", "mk_attn_error_string", "mk_attn_check_status", "mk_attn_version")
+EXPORTED = ("mk_attn_fwd", "mk_attn_fwd_stall_test", "mk_attn_error_string",
+            "mk_attn_check_status", "mk_attn_version")
 
 _lock = threading.Lock()
 _lib = None
@@ -51,6 +52,8 @@ def load_library() -> ctypes.CDLL:
             lib.mk_attn_fwd.argtypes = [vp, vp, vp, vp, vp, i, i, i, i, i, i, ctypes.c_float,
                                         vp, vp]
             lib.mk_attn_fwd.restype = i
+            lib.mk_attn_fwd_stall_test.argtypes = lib.mk_attn_fwd.argtypes
+            lib.mk_attn_fwd_stall_test.restype = i
             lib.mk_attn_error_string.argtypes = [i]
             lib.mk_attn_error_string.restype = ctypes.c_char_p
             lib.mk_attn_check_status.argtypes = [vp]
@@ -66,6 +69,14 @@ def mk_attn_fwd(q: int, k: int, v: int, o: int, lse: int, B: int, Hq: int, Hkv: 
     """Raw C-ABI call: integer device pointers in, status code out."""
     return load_library().mk_attn_fwd(q, k, v, o, lse, B, Hq, Hkv, S, D, int(causal),
                                       float(scale), cu_seqlens, stream)
+
+
+def mk_attn_fwd_stall_test(q: int, k: int, v: int, o: int, lse: int, B: int, Hq: int, Hkv: int,
+                           S: int, D: int, causal: int, scale: float, cu_seqlens: int | None,
+                           stream: int | None) -> int:
+    """Raw C-ABI call of the failure-path test entry (a kernel wait runs out)."""
+    return load_library().mk_attn_fwd_stall_test(q, k, v, o, lse, B, Hq, Hkv, S, D, int(causal),
+                                                 float(scale), cu_seqlens, stream)
 
 
 def mk_attn_error_string(status: int) -> str:

@@ -105,6 +105,7 @@ struct Params {
   int n_units;              // fixed: exact; varlen: upper bound
   float scale_log2;         // scale * log2(e)
   int o_align32;            // o is 32-byte aligned: 256-bit stores in the epilogue
+  int stall_first_slot;     // failure-path test: the CTA's first K/V slot is never signalled
 };
 
 struct Unit {
@@ -301,7 +302,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int s = it % NS;
           ok = mbar_wait_all(&ctl->bar_kv_empty[s], ((it / NS) & 1) ^ 1, abort);
           if (!ok) break;
-          if (elect_one()) {
+          // Failure-path test: iteration 0 is never armed, so the MMA warp's
+          // bounded wait on it runs out and the CTA unwinds with a timeout.
+          if (elect_one() && !(p.stall_first_slot && it == 0)) {
             const uint32_t bytes = (j < n_blk ? C::kTileBytes : 0) + (j > 0 ? C::kTileBytes : 0);
             mbar_arrive_expect_tx(&ctl->bar_kv_full[s], bytes);
             if (j < n_blk) {
@@ -328,7 +331,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (q_iter > 0)
         for (int x = 0; x < 2; ++x) drain_wait(&ctl->bar_q_full[x], (q_iter - 1) & 1);
       for (uint32_t n = (it > (uint32_t)NS ? it - NS : 0); n < it; ++n)
-        drain_wait(&ctl->bar_kv_full[n % NS], (n / NS) & 1);
+        if (!(p.stall_first_slot && n == 0)) drain_wait(&ctl->bar_kv_full[n % NS], (n / NS) & 1);
     } else if (warp == kMmaWarp) {
       // ---------------------------------------------------------- MMA issuer
       constexpr uint32_t idesc_qk = idesc_bf16_f32(kTile, kTile, false, false);
@@ -738,12 +741,10 @@ static int launch(const void *q, const void *k, const void *v, const Params &p, 
 
 }  // namespace mk
 
-extern "C" {
-
-int mk_attn_fwd(const void *q, const void *k, const void *v, void *o, float *lse, int B,
-                int Hq, int Hkv, int S, int D, int causal, float scale,
-                const int32_t *cu_seqlens, void *stream) {
-  using namespace mk;
+namespace mk {
+static int attn_fwd_impl(const void *q, const void *k, const void *v, void *o, float *lse, int B,
+                         int Hq, int Hkv, int S, int D, int causal, float scale,
+                         const int32_t *cu_seqlens, void *stream, int stall_first_slot) {
   if (!q || !k || !v || !o || !lse) return MK_ERR_INVALID_ARG;
   if (B < 1 || Hq < 1 || Hkv < 1 || S < 1) return MK_ERR_INVALID_ARG;
   if (Hq % Hkv != 0) return MK_ERR_INVALID_ARG;
@@ -780,8 +781,24 @@ int mk_attn_fwd(const void *q, const void *k, const void *v, void *o, float *lse
   p.n_units = (int)n_units;
   p.scale_log2 = scale * 1.4426950408889634f;
   p.o_align32 = (reinterpret_cast<uintptr_t>(o) & 31u) == 0;
+  p.stall_first_slot = stall_first_slot;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   return D == 128 ? launch<128>(q, k, v, p, tokens, st) : launch<64>(q, k, v, p, tokens, st);
+}
+}  // namespace mk
+
+extern "C" {
+
+int mk_attn_fwd(const void *q, const void *k, const void *v, void *o, float *lse, int B,
+                int Hq, int Hkv, int S, int D, int causal, float scale,
+                const int32_t *cu_seqlens, void *stream) {
+  return mk::attn_fwd_impl(q, k, v, o, lse, B, Hq, Hkv, S, D, causal, scale, cu_seqlens, stream, 0);
+}
+
+int mk_attn_fwd_stall_test(const void *q, const void *k, const void *v, void *o, float *lse,
+                           int B, int Hq, int Hkv, int S, int D, int causal, float scale,
+                           const int32_t *cu_seqlens, void *stream) {
+  return mk::attn_fwd_impl(q, k, v, o, lse, B, Hq, Hkv, S, D, causal, scale, cu_seqlens, stream, 1);
 }
 
 const char *mk_attn_error_string(int status) {
@@ -809,6 +826,6 @@ int mk_attn_check_status(void *stream) {
   return MK_OK;
 }
 
-int mk_attn_version(void) { return 200; }
+int mk_attn_version(void) { return 300; }
 
 }  // extern "C"
