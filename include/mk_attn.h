@@ -86,10 +86,10 @@ MK_API int mk_attn_fwd(const void *q, const void *k, const void *v, void *o, flo
 
 /*
  * mk_attn_fwd_stall_test -- test support for the failure path only.  Same
- * arguments, checks and return value as mk_attn_fwd, but every CTA leaves its
- * first K/V pipeline slot unsignalled: the kernel's bounded wait on that slot
- * runs out (about 2 s), all roles of the CTA unwind (in-flight copies and
- * MMAs are drained, tensor memory is freed), o and lse are left incomplete,
+ * arguments, checks and return value as mk_attn_fwd, but no CTA loads its
+ * first query tile: the kernel's bounded wait for it runs out (about 2 s), all
+ * roles of the CTA unwind (in-flight copies and MMAs are drained, tensor
+ * memory is freed), o and lse are left incomplete,
  * and the next mk_attn_check_status on the stream returns MK_ERR_TIMEOUT.
  * No fault is raised; the CUDA context stays usable.  Never needed for
  * computing attention.

@@ -105,7 +105,7 @@ struct Params {
   int n_units;              // fixed: exact; varlen: upper bound
   float scale_log2;         // scale * log2(e)
   int o_align32;            // o is 32-byte aligned: 256-bit stores in the epilogue
-  int stall_first_slot;     // failure-path test: the CTA's first K/V slot is never signalled
+  int stall_first_slot;     // failure-path test: the producer loads nothing
 };
 
 struct Unit {
@@ -275,7 +275,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t pol_q = l2_policy_evict_first();
       const uint64_t pol_kv = l2_policy_evict_last();
       uint32_t q_iter = 0, it = 0;
-      bool ok = true;
+      // Failure-path test: the producer issues nothing, so the MMA warp's
+      // bounded wait for the first Q tile runs out and the CTA unwinds.
+      bool ok = !p.stall_first_slot;
       for (int k = 0; ok && k * (int)gridDim.x < p.n_units; ++k) {
         const int u = unit_of_round(k);
         if (u >= p.n_units) continue;
@@ -302,9 +304,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int s = it % NS;
           ok = mbar_wait_all(&ctl->bar_kv_empty[s], ((it / NS) & 1) ^ 1, abort);
           if (!ok) break;
-          // Failure-path test: iteration 0 is never armed, so the MMA warp's
-          // bounded wait on it runs out and the CTA unwinds with a timeout.
-          if (elect_one() && !(p.stall_first_slot && it == 0)) {
+          if (elect_one()) {
             const uint32_t bytes = (j < n_blk ? C::kTileBytes : 0) + (j > 0 ? C::kTileBytes : 0);
             mbar_arrive_expect_tx(&ctl->bar_kv_full[s], bytes);
             if (j < n_blk) {
@@ -331,7 +331,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (q_iter > 0)
         for (int x = 0; x < 2; ++x) drain_wait(&ctl->bar_q_full[x], (q_iter - 1) & 1);
       for (uint32_t n = (it > (uint32_t)NS ? it - NS : 0); n < it; ++n)
-        if (!(p.stall_first_slot && n == 0)) drain_wait(&ctl->bar_kv_full[n % NS], (n / NS) & 1);
+        drain_wait(&ctl->bar_kv_full[n % NS], (n / NS) & 1);
     } else if (warp == kMmaWarp) {
       // ---------------------------------------------------------- MMA issuer
       constexpr uint32_t idesc_qk = idesc_bf16_f32(kTile, kTile, false, false);
