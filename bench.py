@@ -237,6 +237,23 @@ def cpu_oracle_sample(inp, seconds: float, seed: int):
 
 # ------------------------------------------------------------------ our arm
 
+def max_over_ranks(value: float, world: int, device) -> float:
+    """The maximum of `value` over all ranks: the slowest replica sets the job
+    time.  `device` is where the collective's tensor lives (the GPU under
+    NCCL, the CPU under gloo)."""
+    if world <= 1:
+        return value
+    import torch
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tflops(flops_per_rank: float, steps: int, job_ms: float, world: int) -> float:
+    """Whole-job throughput: every rank's FLOPs over the slowest rank's time."""
+    return world * flops_per_rank * steps / (job_ms * 1e-3) / 1e12
+
+
 def run_ours(args, rank: int, world: int, local_rank: int):
     import numpy as np
     import torch
@@ -299,13 +316,9 @@ def run_ours(args, rank: int, world: int, local_rank: int):
         remeasured = True
     if mk_attn_check_status(stream.cuda_stream) != 0:
         raise RuntimeError("kernel reported a timeout in the timed region")
-    total_ms = sum(ms)
-    if world > 1:
-        t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(sum(ms), world, dev)
     ms_per_step = total_ms / args.steps
-    tflops_job = world * flops * args.steps / (total_ms * 1e-3) / 1e12
+    tflops_job = job_tflops(flops, args.steps, total_ms, world)
     per_launch_tflops = flops / (ms_per_step * 1e-3) / 1e12
 
     # End to end through the public API: pinned host inputs -> device, the
@@ -341,12 +354,8 @@ def run_ours(args, rank: int, world: int, local_rank: int):
         e2e_step()
     e1.record(stream)
     torch.cuda.synchronize(dev)
-    e2e_ms = e0.elapsed_time(e1)
-    if world > 1:
-        t = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        e2e_ms = float(t.item())
-    e2e_tflops = world * flops * args.steps / (e2e_ms * 1e-3) / 1e12
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    e2e_tflops = job_tflops(flops, args.steps, e2e_ms, world)
 
     if rank != 0:
         return None
