@@ -82,6 +82,14 @@ struct KernelCfg {
   static constexpr int kSmemBytes = kOffCtl + 512 + 1024;  // + control block + alignment slack
 };
 
+struct Unit {
+  int valid;
+  int b, hq, pair;
+  int seq_start, len;
+};
+
+constexpr int kUnitRing = 4;  // unit descriptors published by the producer warp
+
 struct SharedCtl {
   uint64_t bar_q_full[2], bar_q_empty[2];
   uint64_t bar_kv_full[4], bar_kv_empty[4];  // K/V slots
@@ -89,6 +97,13 @@ struct SharedCtl {
   uint64_t bar_p_full[2][2];  // [tile][half]: P_X keys 0..63, then keys 64..127
   uint64_t bar_o_final[2];
   uint64_t bar_mma_drained;
+  // The producer maps each of the CTA's units once and publishes it here; the
+  // MMA and softmax warps read it.  The producer is at most two units ahead of
+  // the slowest reader (it loads a unit's Q only after the MMA warp has issued
+  // the previous unit's last S, which needs the softmax's last P of the unit
+  // before that), so four entries are never overwritten while still unread.
+  uint64_t bar_unit[kUnitRing];
+  Unit unit_ring[kUnitRing];  // valid = 0: no more units
   uint32_t tmem_base;
   int abort;
 };
@@ -108,18 +123,13 @@ struct Params {
   int stall_first_slot;     // failure-path test: the producer loads nothing
 };
 
-struct Unit {
-  int valid;
-  int b, hq, pair;
-  int seq_start, len;
-};
-
 __device__ __forceinline__ int clamp_tok(int x, int T) { return x < 0 ? 0 : (x > T ? T : x); }
 
 __device__ __forceinline__ int pairs_of_len(int L) { return ((L + kTile - 1) / kTile + 1) / 2; }
 
 // Maps unit index u to (sequence, query head, tile pair).  Must be called by
 // all 32 lanes of a warp (varlen uses a warp scan); every lane gets the result.
+// Only the producer warp maps units; the other roles read its unit ring.
 // Fixed length: units are ordered by pair, heaviest first when causal, so that
 // the static round-robin over CTAs approximates longest-processing-time order;
 // consecutive units share a K/V head (GQA groups are contiguous).  Varlen: unit
@@ -240,6 +250,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&ctl->bar_kv_empty[s], 1);
     }
     mbar_init(&ctl->bar_mma_drained, 1);
+    for (int e = 0; e < kUnitRing; ++e) mbar_init(&ctl->bar_unit[e], 1);
     ctl->abort = 0;
     fence_mbar_init();
   }
@@ -274,15 +285,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       const uint64_t pol_q = l2_policy_evict_first();
       const uint64_t pol_kv = l2_policy_evict_last();
-      uint32_t q_iter = 0, it = 0;
-      // Failure-path test: the producer issues nothing, so the MMA warp's
-      // bounded wait for the first Q tile runs out and the CTA unwinds.
-      bool ok = !p.stall_first_slot;
+      uint32_t q_iter = 0, it = 0, n_pub = 0;
+      auto publish = [&](const Unit &w) {
+        const int e = n_pub % kUnitRing;
+        if (elect_one()) {
+          ctl->unit_ring[e] = w;
+          mbar_arrive(&ctl->bar_unit[e]);  // release: the entry is visible to the waiters
+        }
+        __syncwarp();
+        ++n_pub;
+      };
+      bool ok = true;
       for (int k = 0; ok && k * (int)gridDim.x < p.n_units; ++k) {
         const int u = unit_of_round(k);
         if (u >= p.n_units) continue;
         const Unit w = map_unit(p, cu_smem, u);
         if (!w.valid) continue;
+        publish(w);
+        // Failure-path test: the first unit is published but nothing is
+        // loaded, so the MMA warp's bounded wait for its Q runs out.
+        if (p.stall_first_slot) break;
         const int hkv = w.hq / p.group;
         const int n_blk = max(tile_blocks(p, w, 0), tile_blocks(p, w, 1));
         for (int x = 0; x < 2; ++x) {
@@ -325,6 +347,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();
           ++it;
         }
+      }
+      {
+        const Unit none = {};
+        publish(none);
       }
       // Teardown: every load issued must land before the CTA exits.  For each
       // slot the last issued phase is waited for (earlier phases precede it).
@@ -377,11 +403,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       };
 
-      for (int k = 0; ok && k * (int)gridDim.x < p.n_units; ++k) {
-        const int u = unit_of_round(k);
-        if (u >= p.n_units) continue;
-        const Unit w = map_unit(p, cu_smem, u);
-        if (!w.valid) continue;
+      for (uint32_t n_read = 0; ok; ++n_read) {
+        ok = mbar_wait_all(&ctl->bar_unit[n_read % kUnitRing], (n_read / kUnitRing) & 1, abort);
+        if (!ok) break;
+        const Unit w = ctl->unit_ring[n_read % kUnitRing];
+        if (!w.valid) break;
         const int nx[2] = {tile_blocks(p, w, 0), tile_blocks(p, w, 1)};
         const int n_blk = max(nx[0], nx[1]);
         for (int x = 0; x < 2 && ok; ++x)
@@ -487,11 +513,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t s_cnt = 0, o_cnt = 0;
     bool ok = true;
 
-    for (int k = 0; ok && k * (int)gridDim.x < p.n_units; ++k) {
-        const int u = unit_of_round(k);
-        if (u >= p.n_units) continue;
-      const Unit w = map_unit(p, cu_smem, u);
-      if (!w.valid) continue;
+    for (uint32_t n_read = 0; ok; ++n_read) {
+      ok = mbar_wait_all(&ctl->bar_unit[n_read % kUnitRing], (n_read / kUnitRing) & 1, abort);
+      if (!ok) break;
+      const Unit w = ctl->unit_ring[n_read % kUnitRing];
+      if (!w.valid) break;
       const int n_blk = tile_blocks(p, w, X);
       if (n_blk == 0) continue;
       const int qt = 2 * w.pair + X;
