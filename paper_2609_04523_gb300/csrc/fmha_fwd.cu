@@ -65,6 +65,8 @@ constexpr uint32_t kColS = 0;         // S_X at kColS + 128 * X
 constexpr uint32_t kColO = 256;       // O_X at kColO + D * X
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: rescale O when m rises by > 2^8
 constexpr int kCuCache = 2048;        // cu_seqlens entries cached in shared memory
+constexpr int kMaxLevels = 1024;      // causal varlen: longest-first order up to 1024 tile pairs
+                                      // (262144 tokens) per sequence
 
 __device__ int g_status = 0;               // MK_ERR_TIMEOUT once a wait ran out
 
@@ -78,7 +80,8 @@ struct KernelCfg {
   static constexpr int kOffK = 2 * kTileBytes;
   static constexpr int kOffV = kOffK + kStages * kTileBytes;
   static constexpr int kOffCu = kOffV + kStages * kTileBytes;
-  static constexpr int kOffCtl = kOffCu + kCuCache * 4;
+  static constexpr int kOffLvl = kOffCu + kCuCache * 4;  // (kMaxLevels + 2) ints
+  static constexpr int kOffCtl = kOffLvl + ((kMaxLevels + 2) * 4 + 15) / 16 * 16;
   static constexpr int kSmemBytes = kOffCtl + 512 + 1024;  // + control block + alignment slack
 };
 
@@ -106,6 +109,8 @@ struct SharedCtl {
   Unit unit_ring[kUnitRing];  // valid = 0: no more units
   uint32_t tmem_base;
   int abort;
+  int lvl_P;   // causal varlen: most tile pairs of any sequence
+  int lvl_ok;  // causal varlen: the longest-first level table is valid
 };
 static_assert(sizeof(SharedCtl) <= 512, "control block");
 
@@ -127,17 +132,41 @@ __device__ __forceinline__ int clamp_tok(int x, int T) { return x < 0 ? 0 : (x >
 
 __device__ __forceinline__ int pairs_of_len(int L) { return ((L + kTile - 1) / kTile + 1) / 2; }
 
+// Token range [s0, s1) of varlen sequence b; cu_seqlens entries are clamped
+// to [0, T] and a negative length reads as zero.
+__device__ __forceinline__ void seq_bounds(const Params &p, const int *cu_smem, int b, int &s0,
+                                           int &s1) {
+  const int T = p.S;
+  s0 = clamp_tok(b < kCuCache ? cu_smem[b] : p.cu_seqlens[b], T);
+  s1 = clamp_tok(b + 1 < kCuCache ? cu_smem[b + 1] : p.cu_seqlens[b + 1], T);
+  if (s1 < s0) s1 = s0;
+}
+
+// Causal varlen schedule table (shared memory), for longest-first order: with
+// N(k) = number of sequences with at least k tile pairs and P the most pairs
+// of any sequence, lvl[k] = M(k) = N(k) + N(k+1) + ... + N(P) for k = 1..P+1.
+// Level k (k = P first, down to 1) holds pair k-1 of every sequence with at
+// least k pairs, for every head: Hq * N(k) units, the unit cost growing with k.
+struct Sched {
+  const int *lvl;
+  int P;
+  int ok;
+};
+
 // Maps unit index u to (sequence, query head, tile pair).  Must be called by
-// all 32 lanes of a warp (varlen uses a warp scan); every lane gets the result.
+// all 32 lanes of a warp (varlen uses warp ballots); every lane gets the result.
 // Only the producer warp maps units; the other roles read its unit ring.
 // Fixed length: units are ordered by pair, heaviest first when causal, so that
 // the static round-robin over CTAs approximates longest-processing-time order;
-// consecutive units share a K/V head (GQA groups are contiguous).  Varlen: unit
-// u is pair `u / Hq` of head u % Hq in sequence order; cu_seqlens entries are
-// clamped to [0, T] and negative lengths read as zero.
-__device__ __forceinline__ Unit map_unit(const Params &p, const int *cu_smem, int u) {
+// consecutive units share a K/V head (GQA groups are contiguous).  Causal
+// varlen with a valid table: levels k = P .. 1 in turn, each in sequence order
+// then head order, which again puts the heaviest units first.  Otherwise varlen
+// unit u is pair u / Hq of head u % Hq in sequence order.
+template <bool VL>
+__device__ __forceinline__ Unit map_unit(const Params &p, const int *cu_smem, const Sched &sc,
+                                         int u) {
   Unit w;
-  if (!p.varlen) {
+  if constexpr (!VL) {
     const int per_level = p.B * p.Hq;
     const int level = u / per_level;
     const int rem = u - level * per_level;
@@ -148,21 +177,52 @@ __device__ __forceinline__ Unit map_unit(const Params &p, const int *cu_smem, in
     w.seq_start = w.b * p.S;
     w.len = p.S;
     return w;
-  }
+  } else {
   const int lane = lane_id();
-  const int rank = u / p.Hq;
-  const int T = p.S;
-  w.hq = u % p.Hq;
   w.valid = 0;
-  w.b = w.pair = w.seq_start = w.len = 0;
+  w.b = w.pair = w.seq_start = w.len = w.hq = 0;
+  if (sc.ok) {
+    // Level k: the largest k in [1, P] with Hq * M(k) > u (M is non-increasing).
+    const int64_t uu = u;
+    if (sc.P < 1 || uu >= (int64_t)p.Hq * sc.lvl[1]) return w;
+    int lo = 1, hi = sc.P;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if ((int64_t)p.Hq * sc.lvl[mid] > uu) lo = mid; else hi = mid - 1;
+    }
+    const int k = lo;
+    const int64_t rem = uu - (int64_t)p.Hq * sc.lvl[k + 1];
+    int i = (int)(rem / p.Hq);  // the i-th sequence (in order) with at least k pairs
+    w.hq = (int)(rem - (int64_t)i * p.Hq);
+    w.pair = k - 1;
+    for (int base = 0; base < p.B; base += 32) {
+      const int b = base + lane;
+      int s0 = 0, s1 = 0;
+      if (b < p.B) seq_bounds(p, cu_smem, b, s0, s1);
+      const unsigned m = __ballot_sync(0xffffffffu, b < p.B && pairs_of_len(s1 - s0) >= k);
+      const int c = __popc(m);
+      if (i < c) {
+        unsigned mm = m;
+        for (int t = 0; t < i; ++t) mm &= mm - 1;  // drop the i lowest set bits
+        const int src = __ffs(mm) - 1;
+        w.valid = 1;
+        w.b = base + src;
+        w.seq_start = __shfl_sync(0xffffffffu, s0, src);
+        w.len = __shfl_sync(0xffffffffu, s1 - s0, src);
+        break;
+      }
+      i -= c;
+    }
+    return w;
+  }
+  const int rank = u / p.Hq;
+  w.hq = u % p.Hq;
   int carry = 0;
   for (int base = 0; base < p.B; base += 32) {
     const int b = base + lane;
     int s0 = 0, s1 = 0, np = 0;
     if (b < p.B) {
-      s0 = clamp_tok(b < kCuCache ? cu_smem[b] : p.cu_seqlens[b], T);
-      s1 = clamp_tok(b + 1 < kCuCache ? cu_smem[b + 1] : p.cu_seqlens[b + 1], T);
-      if (s1 < s0) s1 = s0;
+      seq_bounds(p, cu_smem, b, s0, s1);
       np = pairs_of_len(s1 - s0);
     }
     int incl = np;
@@ -186,6 +246,28 @@ __device__ __forceinline__ Unit map_unit(const Params &p, const int *cu_smem, in
     carry += __shfl_sync(0xffffffffu, incl, 31);
   }
   return w;
+  }
+}
+
+// In place, one warp: a[i] = a[i] + a[i+1] + ... + a[n-1] for i in [0, n).
+__device__ __forceinline__ void warp_suffix_sum(int *a, int n) {
+  const int lane = lane_id();
+  const int chunk = (n + 31) / 32;
+  const int lo = lane * chunk, hi = min(n, lo + chunk);
+  int tot = 0;
+  for (int i = hi - 1; i >= lo; --i) {
+    tot += a[i];
+    a[i] = tot;
+  }
+  int incl = tot;  // this lane's chunk and those of the lanes above it
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int y = __shfl_down_sync(0xffffffffu, incl, off);
+    if (lane + off < 32) incl += y;
+  }
+  const int above = incl - tot;
+  for (int i = lo; i < hi; ++i) a[i] += above;
+  __syncwarp();
 }
 
 // Key blocks visited by tile X (0 = A, 1 = B) of a unit; 0 if the tile lies
@@ -213,7 +295,7 @@ __device__ __forceinline__ void drain_wait(uint64_t *bar, uint32_t parity) {
   mbar_wait(bar, parity, &local_abort);
 }
 
-template <int D>
+template <int D, bool VL>
 __global__ void __launch_bounds__(kThreads, 1)
     fmha_fwd_kernel(const __grid_constant__ CUtensorMap tm_q,
                     const __grid_constant__ CUtensorMap tm_k,
@@ -232,9 +314,36 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t sV = smem_addr(smem + C::kOffV);
   const int warp = threadIdx.x / 32;
 
-  if (p.varlen) {
+  int *lvl = reinterpret_cast<int *>(smem + C::kOffLvl);
+  if constexpr (VL) {
     const int n = min(p.B + 1, kCuCache);
     for (int i = threadIdx.x; i < n; i += kThreads) cu_smem[i] = p.cu_seqlens[i];
+  }
+  if (VL && p.causal) {
+    // Longest-first schedule table: a histogram of tile pairs per sequence,
+    // then two suffix sums (see Sched).
+    for (int i = threadIdx.x; i < kMaxLevels + 2; i += kThreads) lvl[i] = 0;
+    if (threadIdx.x == 0) ctl->lvl_P = 0;
+    __syncthreads();
+    for (int b = threadIdx.x; b < p.B; b += kThreads) {
+      int s0, s1;
+      seq_bounds(p, cu_smem, b, s0, s1);
+      const int np = pairs_of_len(s1 - s0);
+      atomicMax(&ctl->lvl_P, np);
+      atomicAdd(&lvl[min(np, kMaxLevels + 1)], 1);
+    }
+    __syncthreads();
+    if (warp == 0) {
+      const int P = ctl->lvl_P;
+      if (P <= kMaxLevels) {
+        warp_suffix_sum(lvl, P + 1);  // lvl[k] = N(k)
+        warp_suffix_sum(lvl, P + 1);  // lvl[k] = M(k); lvl[P + 1] stays 0
+      }
+      if (lane_id() == 0) ctl->lvl_ok = P <= kMaxLevels;
+    }
+  } else if (threadIdx.x == 0) {
+    ctl->lvl_ok = 0;
+    ctl->lvl_P = 0;
   }
   if (threadIdx.x == 0) {
     for (int x = 0; x < 2; ++x) {
@@ -263,6 +372,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after_sync();
   const uint32_t tmem = ctl->tmem_base;
   volatile int *abort = &ctl->abort;
+  const Sched sched = {lvl, ctl->lvl_P, ctl->lvl_ok};
 
   if (warp >= 8) {
     // Third warpgroup: producer, MMA issuer and two idle warps.  All four
@@ -299,7 +409,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int k = 0; ok && k * (int)gridDim.x < p.n_units; ++k) {
         const int u = unit_of_round(k);
         if (u >= p.n_units) continue;
-        const Unit w = map_unit(p, cu_smem, u);
+        const Unit w = map_unit<VL>(p, cu_smem, sched, u);
         if (!w.valid) continue;
         publish(w);
         // Failure-path test: the first unit is published but nothing is
@@ -671,7 +781,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_before_sync();
       if (row_valid) {
         const float lse = (m_run + log2f(l_run)) * 0.69314718055994530942f;
-        const int64_t li = p.varlen ? (int64_t)w.hq * p.S + tok
+        const int64_t li = VL ? (int64_t)w.hq * p.S + tok
                                     : ((int64_t)w.b * p.Hq + w.hq) * p.S + qpos;
         p.lse[li] = lse;
       }
@@ -723,13 +833,25 @@ static bool encode_tokens_heads_dim(CUtensorMap *map, const void *base, uint64_t
 struct DeviceInfo {
   std::once_flag once;
   int sm_count = 0;
-  cudaError_t attr_err[2] = {cudaSuccess, cudaSuccess};
-  int regs[2] = {0, 0};
+  cudaError_t attr_err[4] = {cudaSuccess, cudaSuccess, cudaSuccess, cudaSuccess};
+  int regs[4] = {0, 0, 0, 0};  // [D == 128][varlen]
 };
 
 static DeviceInfo g_devices[64];
 
-template <int D>
+// Sets the shared-memory limit and reads the register count of one kernel
+// instantiation (first call on a device only).
+template <int D, bool VL>
+static void kernel_setup(DeviceInfo &di) {
+  const int vi = (D == 128 ? 2 : 0) + (VL ? 1 : 0);
+  di.attr_err[vi] = cudaFuncSetAttribute(fmha_fwd_kernel<D, VL>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         KernelCfg<D>::kSmemBytes);
+  cudaFuncAttributes fa;
+  if (cudaFuncGetAttributes(&fa, fmha_fwd_kernel<D, VL>) == cudaSuccess) di.regs[vi] = fa.numRegs;
+}
+
+template <int D, bool VL>
 static int launch(const void *q, const void *k, const void *v, const Params &p, int64_t tokens,
                   cudaStream_t stream) {
   using C = KernelCfg<D>;
@@ -744,24 +866,19 @@ static int launch(const void *q, const void *k, const void *v, const Params &p, 
   std::call_once(di.once, [&] {
     if (cudaDeviceGetAttribute(&di.sm_count, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
       di.sm_count = 0;
-    di.attr_err[0] = cudaFuncSetAttribute(fmha_fwd_kernel<64>,
-                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          KernelCfg<64>::kSmemBytes);
-    di.attr_err[1] = cudaFuncSetAttribute(fmha_fwd_kernel<128>,
-                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          KernelCfg<128>::kSmemBytes);
-    cudaFuncAttributes fa;
-    if (cudaFuncGetAttributes(&fa, fmha_fwd_kernel<64>) == cudaSuccess) di.regs[0] = fa.numRegs;
-    if (cudaFuncGetAttributes(&fa, fmha_fwd_kernel<128>) == cudaSuccess) di.regs[1] = fa.numRegs;
+    kernel_setup<64, false>(di);
+    kernel_setup<64, true>(di);
+    kernel_setup<128, false>(di);
+    kernel_setup<128, true>(di);
   });
-  const int vi = D == 128 ? 1 : 0;
+  const int vi = (D == 128 ? 2 : 0) + (VL ? 1 : 0);
   if (di.sm_count <= 0 || di.attr_err[vi] != cudaSuccess) return MK_ERR_CUDA;
   // The warpgroup register split assumes the block launches with exactly
   // kLaunchRegs registers per thread; anything else could leave a
   // setmaxnreg.inc waiting forever, so refuse to launch.
   if (di.regs[vi] != kLaunchRegs) return MK_ERR_CUDA;
   const int grid = p.n_units < di.sm_count ? p.n_units : di.sm_count;
-  fmha_fwd_kernel<D><<<grid, kThreads, C::kSmemBytes, stream>>>(tq, tk, tv, p);
+  fmha_fwd_kernel<D, VL><<<grid, kThreads, C::kSmemBytes, stream>>>(tq, tk, tv, p);
   return cudaGetLastError() == cudaSuccess ? MK_OK : MK_ERR_CUDA;
 }
 
@@ -809,7 +926,9 @@ static int attn_fwd_impl(const void *q, const void *k, const void *v, void *o, f
   p.o_align32 = (reinterpret_cast<uintptr_t>(o) & 31u) == 0;
   p.stall_first_slot = stall_first_slot;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  return D == 128 ? launch<128>(q, k, v, p, tokens, st) : launch<64>(q, k, v, p, tokens, st);
+  if (D == 128)
+    return varlen ? launch<128, true>(q, k, v, p, tokens, st) : launch<128, false>(q, k, v, p, tokens, st);
+  return varlen ? launch<64, true>(q, k, v, p, tokens, st) : launch<64, false>(q, k, v, p, tokens, st);
 }
 }  // namespace mk
 
