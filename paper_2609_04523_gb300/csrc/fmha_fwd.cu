@@ -12,9 +12,15 @@
 //   warps 0-3   softmax of tile A, thread r owns row r = TMEM lane r
 //   warps 4-7   softmax of tile B (same lanes, warp % 4 selects the lane quarter)
 //   warp 8      tcgen05 MMA issuer (one thread)
-//   warp 9      TMA producer (one thread): Q_A, Q_B per unit, then K_j, V_j
-//               blocks of 128 keys through an n-stage 128-byte-swizzled ring
+//   warp 9      TMA producer (one thread): maps each of the CTA's units once
+//               and publishes it in a small shared-memory ring for the other
+//               roles; Q_A, Q_B per unit, then K_j, V_j blocks of 128 keys
+//               through an n-stage 128-byte-swizzled ring
 //   warps 10-11 idle (they complete the third warpgroup)
+// Schedule: units are dealt to the persistent CTAs round by round (snake
+// order), heaviest first: fixed length by tile pair, causal varlen by level
+// (pair index) from a per-CTA table, which approximates longest-processing-
+// time order.  Fixed length and varlen are separate instantiations.
 // Registers: the block launches with 168 per thread (384 threads); the third
 // warpgroup gives back down to kRegsCtl and the two softmax warpgroups grow to
 // kRegsSoftmax, so each SM sub-partition (one warp of each warpgroup) stays
