@@ -623,6 +623,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t t_row = tmem + ((uint32_t)((warp % 4) * 32) << 16);
     const uint32_t t_s = t_row + kColS + X * 128;
     const uint32_t t_o = t_row + kColO + X * D;
+    // o is written once and not read again by this kernel: its lines go first
+    // when L2 needs room, so the K/V blocks other query tiles still read stay.
+    const uint64_t pol_o = l2_policy_evict_first();
     const float c2 = p.scale_log2;
     const bool neg_scale = c2 < 0.f;
     const float c2a = fmaxf(fabsf(c2), 1.17549435e-38f);  // |c2|, at least FLT_MIN
@@ -773,12 +776,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           // Each thread writes its own row: 32-byte stores fill whole sectors
           // (half as many store instructions and sector writes as 16-byte ones).
           if (p.o_align32) {
-            st_global_v8(dst + c * 4, v[0], v[1], v[2], v[3], v[4], v[5], v[6], v[7]);
-            st_global_v8(dst + c * 4 + 2, v[8], v[9], v[10], v[11], v[12], v[13], v[14], v[15]);
+            st_global_v8_hint(dst + c * 4, v[0], v[1], v[2], v[3], v[4], v[5], v[6], v[7], pol_o);
+            st_global_v8_hint(dst + c * 4 + 2, v[8], v[9], v[10], v[11], v[12], v[13], v[14], v[15],
+                              pol_o);
           } else {
 #pragma unroll
             for (int e = 0; e < 4; ++e)
-              dst[c * 4 + e] = make_uint4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
+              st_global_v4_hint(dst + c * 4 + e, v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3],
+                                pol_o);
           }
         }
       }

@@ -303,6 +303,24 @@ __device__ __forceinline__ void st_global_v8(void *ptr, uint32_t a0, uint32_t a1
                : "memory");
 }
 
+// As st_global_v8, with an L2 cache policy (from createpolicy).
+__device__ __forceinline__ void st_global_v8_hint(void *ptr, uint32_t a0, uint32_t a1,
+                                                  uint32_t a2, uint32_t a3, uint32_t a4,
+                                                  uint32_t a5, uint32_t a6, uint32_t a7,
+                                                  uint64_t policy) {
+  asm volatile("st.global.L2::cache_hint.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8}, %9;" ::"l"(ptr),
+               "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(a4), "r"(a5), "r"(a6), "r"(a7), "l"(policy)
+               : "memory");
+}
+
+// As a 16-byte store, with an L2 cache policy (from createpolicy).
+__device__ __forceinline__ void st_global_v4_hint(void *ptr, uint32_t a0, uint32_t a1,
+                                                  uint32_t a2, uint32_t a3, uint64_t policy) {
+  asm volatile("st.global.L2::cache_hint.v4.b32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(ptr), "r"(a0),
+               "r"(a1), "r"(a2), "r"(a3), "l"(policy)
+               : "memory");
+}
+
 // ------------------------------------------------------------------ scalars
 
 // 2^x on the MUFU unit (approximate, flush-to-zero; 2^-inf = +0).
