@@ -63,6 +63,9 @@ def _bind(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.mk_oracle_attn_rows_f64.argtypes = [p, p, p, i, i, i, i, i, i, ctypes.c_double,
                                             p, p, ctypes.c_int64, p, p, i]
     lib.mk_oracle_attn_rows_f64.restype = i
+    lib.mk_oracle_decode_paged_f64.argtypes = [p, p, p, p, p, p, p, i, i, i, i, i, i, i,
+                                               ctypes.c_double, i]
+    lib.mk_oracle_decode_paged_f64.restype = i
     return lib
 
 
@@ -159,4 +162,28 @@ def attn_rows(q, k, v, causal: bool, scale: float, rows, cu_seqlens=None,
                                      n, _ptr(o), _ptr(lse), int(n_threads or default_threads()))
     if st != 0:
         raise ValueError(f"oracle rejected the rows (status {st})")
+    return o, lse
+
+
+def decode_paged(q, k_cache, v_cache, page_table, seq_lens, scale: float,
+                 n_threads: int | None = None, lib: ctypes.CDLL | None = None):
+    """One decode step against a paged K/V cache, in fp64.
+
+    q: [B,Hq,D]; k_cache/v_cache: [num_pages, page_size, Hkv, D] (bf16 tensors
+    or uint16 bit arrays); page_table: int32 [B, max_pages]; seq_lens: int32
+    [B].  Returns (o [B,Hq,D], lse [B,Hq]) as fp64 numpy arrays."""
+    qb, kb, vb = _bits(q), _bits(k_cache), _bits(v_cache)
+    pt = np.ascontiguousarray(np.asarray(page_table, dtype=np.int32))
+    sl = np.ascontiguousarray(np.asarray(seq_lens, dtype=np.int32))
+    B, Hq, D = qb.shape
+    num_pages, page_size, Hkv, _ = kb.shape
+    o = np.zeros((B, Hq, D), dtype=np.float64)
+    lse = np.zeros((B, Hq), dtype=np.float64)
+    lib = lib or load()
+    st = lib.mk_oracle_decode_paged_f64(_ptr(qb), _ptr(kb), _ptr(vb), _ptr(pt), _ptr(sl),
+                                        _ptr(o), _ptr(lse), B, Hq, Hkv, D, page_size,
+                                        pt.shape[1], num_pages, float(scale),
+                                        int(n_threads or default_threads()))
+    if st != 0:
+        raise ValueError(f"oracle rejected the decode problem (status {st})")
     return o, lse

@@ -303,3 +303,116 @@ int mk_oracle_attn_rows_f64(const uint16_t *q, const uint16_t *k, const uint16_t
     rows_job_t job = {&p, rows, o_rows, lse_rows, n_rows, &next, max_seq_len(&p)};
     return run_threads(rows_worker, &job, sizeof job, n_threads);
 }
+
+/* ------------------------------------------------------ paged decode step */
+
+/*
+ * One decode step against a paged key/value cache: for each sequence b, its
+ * newest query q[b,h,:] attends to the L_b = seq_lens[b] cached positions
+ * 0..L_b-1 of that sequence (all of them: the new token is the last
+ * position, so no causal mask applies).  Position j lives in physical page
+ * page_table[b * max_pages + j / page_size], slot j % page_size:
+ *
+ *   k_j  = k_cache[page, slot, g, :],  v_j = v_cache[page, slot, g, :]
+ *   s_j  = scale * sum_d q[b,h,d] * k_j[d]          (g = h / (Hq / Hkv))
+ *   o[d] = sum_j exp(s_j - m) v_j[d] / sum_j exp(s_j - m),  m = max_j s_j
+ *   lse  = m + ln(sum_j exp(s_j - m))
+ *
+ * This is the attention definition above, for a single query row whose key
+ * set is gathered through a page table (the Paged Attention row of Table 2).
+ * Layouts: q, o [B, Hq, D]; k_cache, v_cache [num_pages, page_size, Hkv, D];
+ * page_table int32 [B, max_pages]; seq_lens int32 [B]; lse [B, Hq].
+ * L_b = 0 gives o = 0 and lse = -inf.  Returns MK_ORACLE_BAD_ARG for sizes
+ * out of range, a length above max_pages * page_size, or a page index
+ * outside [0, num_pages).
+ */
+typedef struct {
+    const uint16_t *q, *kc, *vc;
+    const int32_t *page_table, *seq_lens;
+    double *o, *lse;
+    int B, Hq, Hkv, D, page_size, max_pages;
+    double scale;
+    int64_t *next;
+    int max_len;
+} decode_job_t;
+
+static void *decode_worker(void *arg)
+{
+    decode_job_t *job = (decode_job_t *)arg;
+    const int G = job->Hq / job->Hkv, D = job->D;
+    double *s_buf = (double *)malloc(sizeof(double) * (size_t)(job->max_len > 0 ? job->max_len : 1));
+    if (!s_buf)
+        return NULL;
+    for (;;) {
+        int64_t t = __atomic_fetch_add(job->next, 1, __ATOMIC_RELAXED);
+        if (t >= (int64_t)job->B * job->Hq)
+            break;
+        const int b = (int)(t / job->Hq), h = (int)(t % job->Hq), g = h / G;
+        const int L = job->seq_lens[b];
+        const uint16_t *qr = job->q + ((int64_t)b * job->Hq + h) * D;
+        double *orow = job->o + ((int64_t)b * job->Hq + h) * D;
+        for (int d = 0; d < D; ++d)
+            orow[d] = 0.0;
+        if (L == 0) {
+            job->lse[t] = -INFINITY;
+            continue;
+        }
+        double m = -INFINITY;
+        for (int j = 0; j < L; ++j) {
+            const int64_t page = job->page_table[(int64_t)b * job->max_pages + j / job->page_size];
+            const int64_t row = (page * job->page_size + j % job->page_size) * job->Hkv + g;
+            const uint16_t *kr = job->kc + row * D;
+            double acc = 0.0;
+            for (int d = 0; d < D; ++d)
+                acc += bf16_bits_to_f64(qr[d]) * bf16_bits_to_f64(kr[d]);
+            s_buf[j] = job->scale * acc;
+            if (s_buf[j] > m)
+                m = s_buf[j];
+        }
+        double l = 0.0;
+        for (int j = 0; j < L; ++j) {
+            const double e = exp(s_buf[j] - m);
+            l += e;
+            const int64_t page = job->page_table[(int64_t)b * job->max_pages + j / job->page_size];
+            const int64_t row = (page * job->page_size + j % job->page_size) * job->Hkv + g;
+            const uint16_t *vr = job->vc + row * D;
+            for (int d = 0; d < D; ++d)
+                orow[d] += e * bf16_bits_to_f64(vr[d]);
+        }
+        for (int d = 0; d < D; ++d)
+            orow[d] /= l;
+        job->lse[t] = m + log(l);
+    }
+    free(s_buf);
+    return NULL;
+}
+
+int mk_oracle_decode_paged_f64(const uint16_t *q, const uint16_t *k_cache,
+                               const uint16_t *v_cache, const int32_t *page_table,
+                               const int32_t *seq_lens, double *o, double *lse, int B, int Hq,
+                               int Hkv, int D, int page_size, int max_pages, int num_pages,
+                               double scale, int n_threads)
+{
+    if (!q || !k_cache || !v_cache || !page_table || !seq_lens || !o || !lse)
+        return MK_ORACLE_BAD_ARG;
+    if (B < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || D < 1 || page_size < 1 ||
+        max_pages < 1 || num_pages < 1)
+        return MK_ORACLE_BAD_ARG;
+    int max_len = 0;
+    for (int b = 0; b < B; ++b) {
+        const int L = seq_lens[b];
+        if (L < 0 || (int64_t)L > (int64_t)max_pages * page_size)
+            return MK_ORACLE_BAD_ARG;
+        for (int j = 0; j * page_size < L; ++j) {
+            const int32_t pg = page_table[(int64_t)b * max_pages + j];
+            if (pg < 0 || pg >= num_pages)
+                return MK_ORACLE_BAD_ARG;
+        }
+        if (L > max_len)
+            max_len = L;
+    }
+    int64_t next = 0;
+    decode_job_t job = {q, k_cache, v_cache, page_table, seq_lens, o, lse, B, Hq, Hkv, D,
+                        page_size, max_pages, scale, &next, max_len};
+    return run_threads(decode_worker, &job, sizeof job, n_threads);
+}

@@ -244,3 +244,48 @@ def sample_rows(lengths, Hq: int, n: int, seed: int, tile: int = TILE) -> np.nda
         b = int(np.searchsorted(cum, t, side="right") - 1)
         rows.append((b, int(rng.integers(0, Hq)), int(t - cum[b])))
     return np.asarray(rows, dtype=np.int64)
+
+
+# ------------------------------------------------------------ paged decode
+
+@dataclass
+class PagedInputs:
+    """One decode step against a paged K/V cache (see make_paged)."""
+    q: torch.Tensor           # bf16 [B, Hq, D]
+    k_cache: torch.Tensor     # bf16 [num_pages, page_size, Hkv, D]
+    v_cache: torch.Tensor     # bf16 [num_pages, page_size, Hkv, D]
+    page_table: torch.Tensor  # int32 [B, max_pages]
+    seq_lens: torch.Tensor    # int32 [B]
+    scale: float
+
+
+def make_paged(seq_lens, Hq: int, Hkv: int, D: int, page_size: int, seed: int,
+               sigma: float = 1.0, spare_pages: int = 3, max_pages: int | None = None) -> PagedInputs:
+    """Seeded decode inputs: each sequence's ceil(L/page_size) logical pages
+    get distinct physical pages in a random order (with `spare_pages` unused
+    pages mixed in), the way a cache allocator hands them out.  Unused
+    page-table entries are -1.  Pure data generation: no attention arithmetic."""
+    g = torch.Generator("cpu").manual_seed(seed)
+    lens = [int(x) for x in seq_lens]
+    need = [(L + page_size - 1) // page_size for L in lens]
+    mp = max(1, max(need) if max_pages is None else max_pages)
+    num_pages = sum(need) + spare_pages
+    perm = torch.randperm(num_pages, generator=g).tolist()
+    pt = torch.full((len(lens), mp), -1, dtype=torch.int32)
+    at = 0
+    for b, n in enumerate(need):
+        for j in range(n):
+            pt[b, j] = perm[at]
+            at += 1
+    q = randn_bf16((len(lens), Hq, D), g, sigma)
+    kc = randn_bf16((num_pages, page_size, Hkv, D), g, sigma)
+    vc = randn_bf16((num_pages, page_size, Hkv, D), g, sigma)
+    return PagedInputs(q, kc, vc, pt, torch.tensor(lens, dtype=torch.int32), 1.0 / math.sqrt(D))
+
+
+def decode_bytes(seq_lens, Hq: int, Hkv: int, D: int) -> int:
+    """Minimal HBM traffic of one decode step: every cached key and value of
+    every sequence read once, q read and o written once (bf16), lse written."""
+    keys = int(sum(int(x) for x in seq_lens))
+    B = len(seq_lens)
+    return 2 * 2 * keys * Hkv * D + 2 * 2 * B * Hq * D + 4 * B * Hq

@@ -306,6 +306,99 @@ def check_rows_match_full(lib):
         _close(lrow[n], lse[h, t], 0.0, "rows vs full lse")
 
 
+# ------------------------------------------------------- paged decode step
+
+def _decode(lib, inp):
+    return oracle.decode_paged(inp.q, inp.k_cache, inp.v_cache, inp.page_table, inp.seq_lens,
+                               inp.scale, n_threads=2, lib=lib)
+
+
+def _gather(cache, page_table, L, page_size):
+    """The first L cached positions of one sequence, contiguous: [L, Hkv, D]."""
+    rows = [cache[int(page_table[j // page_size]), j % page_size] for j in range(L)]
+    return torch.stack(rows) if rows else cache[:0, 0]
+
+
+def check_decode_equals_prefill_last_row(lib):
+    """A decode step is the last row of causal attention over the same keys:
+    gather each sequence's pages into a packed varlen batch, put the decode
+    query at its last position, and ask the (separately pinned) prefill
+    definition for that row."""
+    lens, Hq, Hkv, D, ps = [1, 7, 16, 33, 50], 6, 2, 8, 16
+    inp = W.make_paged(lens, Hq, Hkv, D, ps, seed=140)
+    o, lse = _decode(lib, inp)
+    k = torch.cat([_gather(inp.k_cache, inp.page_table[b], L, ps) for b, L in enumerate(lens)])
+    v = torch.cat([_gather(inp.v_cache, inp.page_table[b], L, ps) for b, L in enumerate(lens)])
+    q = torch.zeros((sum(lens), Hq, D), dtype=torch.bfloat16)
+    starts = np.cumsum([0] + lens)
+    for b, L in enumerate(lens):
+        q[starts[b] + L - 1] = inp.q[b]
+    rows = np.array([(b, h, L - 1) for b, L in enumerate(lens) for h in range(Hq)], dtype=np.int64)
+    o_ref, lse_ref = oracle.attn_rows(q, k, v, True, inp.scale, rows, cu_seqlens=starts,
+                                      n_threads=2, lib=lib)
+    _close(o.reshape(-1, D), o_ref, TIGHT, "decode vs prefill last row o")
+    _close(lse.reshape(-1), lse_ref, TIGHT, "decode vs prefill last row lse")
+
+
+def check_decode_page_permutation(lib):
+    """Where the pages sit in the cache does not matter: relabelling the
+    physical pages (and the page table with them) changes nothing."""
+    lens, Hq, Hkv, D, ps = [40, 3, 64], 4, 4, 8, 8
+    inp = W.make_paged(lens, Hq, Hkv, D, ps, seed=141, spare_pages=5)
+    o, lse = _decode(lib, inp)
+    n = inp.k_cache.shape[0]
+    perm = torch.from_numpy(np.random.default_rng(7).permutation(n))  # new slot of page i
+    inv = torch.empty_like(perm)
+    inv[perm] = torch.arange(n)
+    pt = inp.page_table.clone()
+    pt[pt >= 0] = perm[pt[pt >= 0].long()].int()
+    moved = W.PagedInputs(inp.q, inp.k_cache[inv], inp.v_cache[inv], pt, inp.seq_lens, inp.scale)
+    o2, lse2 = _decode(lib, moved)
+    _close(o, o2, 0.0, "page permutation o")
+    _close(lse, lse2, 0.0, "page permutation lse")
+
+
+def check_decode_single_key(lib):
+    """One cached key: o = v_0 and lse = scale * q . k_0."""
+    Hq, Hkv, D, ps = 4, 2, 16, 16
+    inp = W.make_paged([1, 1], Hq, Hkv, D, ps, seed=142)
+    o, lse = _decode(lib, inp)
+    for b in range(2):
+        pg = int(inp.page_table[b, 0])
+        for h in range(Hq):
+            g = h // (Hq // Hkv)
+            k0 = _f64(inp.k_cache[pg, 0, g])
+            v0 = _f64(inp.v_cache[pg, 0, g])
+            _close(o[b, h], v0, TIGHT, "single key o")
+            _close(lse[b, h], inp.scale * float(np.dot(_f64(inp.q[b, h]), k0)), TIGHT, "single key lse")
+
+
+def check_decode_identical_keys(lib):
+    """All cached keys equal: the weights are uniform, so o is the mean of the
+    values and lse = scale * q . k + ln L."""
+    Hq, Hkv, D, ps, L = 2, 1, 8, 8, 21
+    inp = W.make_paged([L], Hq, Hkv, D, ps, seed=143)
+    kc = inp.k_cache.clone()
+    kc[:] = kc[int(inp.page_table[0, 0]), 0]
+    inp = W.PagedInputs(inp.q, kc, inp.v_cache, inp.page_table, inp.seq_lens, inp.scale)
+    o, lse = _decode(lib, inp)
+    v = _f64(_gather(inp.v_cache, inp.page_table[0], L, ps))[:, 0]
+    k0 = _f64(kc[0, 0, 0])
+    for h in range(Hq):
+        _close(o[0, h], v.mean(axis=0), 1e-12, "identical keys o")
+        _close(lse[0, h], inp.scale * float(np.dot(_f64(inp.q[0, h]), k0)) + math.log(L), 1e-12,
+               "identical keys lse")
+
+
+def check_decode_empty_sequence(lib):
+    """No cached key: o = 0 and lse = -inf (the defensive reading)."""
+    inp = W.make_paged([0, 9], 2, 2, 8, 8, seed=144)
+    o, lse = _decode(lib, inp)
+    assert np.all(o[0] == 0.0), "empty sequence o"
+    assert np.all(np.isneginf(lse[0])), "empty sequence lse"
+    assert np.all(np.isfinite(lse[1])), "non-empty sequence lse"
+
+
 ALL_CHECKS = [
     check_brute_force_tiny,
     check_brute_force_varlen,
@@ -323,4 +416,9 @@ ALL_CHECKS = [
     check_logit_shift,
     check_value_affine,
     check_rows_match_full,
+    check_decode_equals_prefill_last_row,
+    check_decode_page_permutation,
+    check_decode_single_key,
+    check_decode_identical_keys,
+    check_decode_empty_sequence,
 ]

@@ -34,6 +34,12 @@ MUTANTS = {
     "weights_not_accumulated": ("        l += w;\n", "        l = w;\n"),
     "last_dim_dropped": ("for (int d = 0; d < D; ++d)\n            dot +=",
                          "for (int d = 0; d + 1 < D; ++d)\n            dot +="),
+    "decode_slot_from_page_index": (
+        "const int64_t row = (page * job->page_size + j % job->page_size) * job->Hkv + g;\n            const uint16_t *kr",
+        "const int64_t row = (page * job->page_size + j / job->page_size) * job->Hkv + g;\n            const uint16_t *kr"),
+    "decode_interleaved_groups": ("h = (int)(t % job->Hq), g = h / G;", "h = (int)(t % job->Hq), g = h % job->Hkv;"),
+    "decode_drop_scale": ("s_buf[j] = job->scale * acc;", "s_buf[j] = acc;"),
+    "decode_lse_log2": ("job->lse[t] = m + log(l);", "job->lse[t] = m + log2(l);"),
 }
 
 
