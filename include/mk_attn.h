@@ -98,13 +98,67 @@ MK_API int mk_attn_fwd_stall_test(const void *q, const void *k, const void *v, v
                                   float *lse, int B, int Hq, int Hkv, int S, int D, int causal,
                                   float scale, const int32_t *cu_seqlens, void *stream);
 
+/*
+ * mk_attn_decode_workspace_bytes -- bytes of device workspace that
+ * mk_attn_decode_paged needs for these sizes on the current device (0: none),
+ * or -1 for invalid sizes.  Depends on the device's SM count only through the
+ * number of KV splits it chooses.
+ */
+MK_API int64_t mk_attn_decode_workspace_bytes(int B, int Hq, int Hkv, int D, int page_size,
+                                              int max_pages);
+
+/*
+ * mk_attn_decode_paged -- one decode step against a paged key/value cache
+ * (the Paged Attention row of the paper's Table 2).  For each sequence b and
+ * query head h (key/value head h / (Hq/Hkv)), the newest query attends to all
+ * L_b = seq_lens[b] cached positions of its sequence (no mask: the query is
+ * the last position):
+ *   o[b,h,:] = sum_j softmax_j(scale * q[b,h,:] . k_j) v_j
+ *   lse[b,h] = ln sum_j exp(scale * q[b,h,:] . k_j)
+ * where position j is slot j % page_size of physical page
+ * page_table[b, j / page_size].
+ *
+ * Arguments (all pointers are DEVICE pointers owned by the caller):
+ *   q            bf16 [B, Hq, D].  Read only.
+ *   k_cache,     bf16 [num_pages, page_size, Hkv, D].  Read only.
+ *   v_cache
+ *   page_table   int32 [B, max_pages]; entries j < ceil(L_b / page_size)
+ *                must lie in [0, num_pages).  Read only, on the device.
+ *   seq_lens     int32 [B], each in [0, max_pages * page_size].  Read only.
+ *   o            bf16 [B, Hq, D] output, fully overwritten.
+ *   lse          fp32 [B, Hq] output, fully overwritten (natural log, scale
+ *                included); L_b = 0 gives o = 0 and lse = -inf.
+ *   D            64 or 128.   page_size  16, 32, 64 or 128.
+ *   Hq / Hkv     at most 16.
+ *   workspace    device buffer of at least mk_attn_decode_workspace_bytes()
+ *                bytes, 16-byte aligned, or NULL when that is 0.  Scratch
+ *                for the per-split partial results; its contents on entry
+ *                do not matter.  Launches that share a workspace must not
+ *                overlap in time.
+ *   stream       cudaStream_t; the call is asynchronous and never syncs.
+ * Returns MK_OK; MK_ERR_INVALID_ARG (null pointer, sizes out of range, a
+ * missing or too small workspace), MK_ERR_UNSUPPORTED (D, page_size, or a
+ * head group above 16), MK_ERR_ALIGNMENT (q, caches, o or workspace not
+ * 16-byte aligned; page_table, seq_lens or lse not 4-byte aligned), or
+ * MK_ERR_CUDA.  On any error nothing is launched.  Page-table entries or
+ * lengths out of range, which only the device sees, leave o and lse undefined
+ * and make the next mk_attn_check_status return MK_ERR_INVALID_ARG.
+ */
+MK_API int mk_attn_decode_paged(const void *q, const void *k_cache, const void *v_cache,
+                                const int32_t *page_table, const int32_t *seq_lens, void *o,
+                                float *lse, int B, int Hq, int Hkv, int D, int page_size,
+                                int max_pages, int num_pages, float scale, void *workspace,
+                                int64_t workspace_bytes, void *stream);
+
 /* Short static description of a status code.  Never NULL. */
 MK_API const char *mk_attn_error_string(int status);
 
 /*
  * mk_attn_check_status -- synchronises `stream`, then reads and clears the
- * device status word written by kernels whose internal waits ran out.
- * Returns MK_OK, MK_ERR_TIMEOUT, or MK_ERR_CUDA if synchronisation failed.
+ * device status words written by kernels whose internal waits ran out or
+ * that met device-side inputs out of range (decode page tables, lengths).
+ * Returns MK_OK, MK_ERR_TIMEOUT, MK_ERR_INVALID_ARG, or MK_ERR_CUDA if
+ * synchronisation failed.
  */
 MK_API int mk_attn_check_status(void *stream);
 

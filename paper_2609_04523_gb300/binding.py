@@ -21,8 +21,9 @@ MK_ERR_CUDA = -4
 MK_ERR_TIMEOUT = -5
 
 # Symbols declared in include/mk_attn.h.
-EXPORTED = ("mk_attn_fwd", "mk_attn_fwd_stall_test", "mk_attn_error_string",
-            "mk_attn_check_status", "mk_attn_version")
+EXPORTED = ("mk_attn_fwd", "mk_attn_fwd_stall_test", "mk_attn_decode_workspace_bytes",
+            "mk_attn_decode_paged", "mk_attn_error_string", "mk_attn_check_status",
+            "mk_attn_version")
 
 _lock = threading.Lock()
 _lib = None
@@ -54,6 +55,12 @@ def load_library() -> ctypes.CDLL:
             lib.mk_attn_fwd.restype = i
             lib.mk_attn_fwd_stall_test.argtypes = lib.mk_attn_fwd.argtypes
             lib.mk_attn_fwd_stall_test.restype = i
+            i64 = ctypes.c_int64
+            lib.mk_attn_decode_workspace_bytes.argtypes = [i, i, i, i, i, i]
+            lib.mk_attn_decode_workspace_bytes.restype = i64
+            lib.mk_attn_decode_paged.argtypes = [vp, vp, vp, vp, vp, vp, vp, i, i, i, i, i, i, i,
+                                                 ctypes.c_float, vp, i64, vp]
+            lib.mk_attn_decode_paged.restype = i
             lib.mk_attn_error_string.argtypes = [i]
             lib.mk_attn_error_string.restype = ctypes.c_char_p
             lib.mk_attn_check_status.argtypes = [vp]
@@ -143,4 +150,64 @@ def attn_fwd(q, k, v, causal: bool = True, scale: float | None = None, cu_seqlen
     _check(mk_attn_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), lse.data_ptr(),
                        B, Hq, Hkv, S, D, int(bool(causal)), float(scale), cu_ptr,
                        stream.cuda_stream))
+    return out, lse
+
+
+def mk_attn_decode_workspace_bytes(B: int, Hq: int, Hkv: int, D: int, page_size: int,
+                                   max_pages: int) -> int:
+    return load_library().mk_attn_decode_workspace_bytes(B, Hq, Hkv, D, page_size, max_pages)
+
+
+def mk_attn_decode_paged(q: int, k_cache: int, v_cache: int, page_table: int, seq_lens: int,
+                         o: int, lse: int, B: int, Hq: int, Hkv: int, D: int, page_size: int,
+                         max_pages: int, num_pages: int, scale: float, workspace: int | None,
+                         workspace_bytes: int, stream: int | None) -> int:
+    """Raw C-ABI call: integer device pointers in, status code out."""
+    return load_library().mk_attn_decode_paged(q, k_cache, v_cache, page_table, seq_lens, o, lse,
+                                               B, Hq, Hkv, D, page_size, max_pages, num_pages,
+                                               float(scale), workspace, int(workspace_bytes),
+                                               stream)
+
+
+def decode_paged(q, k_cache, v_cache, page_table, seq_lens, scale: float | None = None,
+                 out=None, lse=None, workspace=None, stream=None):
+    """One decode step against a paged K/V cache through mk_attn_decode_paged.
+
+    q: [B,Hq,D] bf16; k_cache/v_cache: [num_pages, page_size, Hkv, D] bf16;
+    page_table: int32 [B, max_pages]; seq_lens: int32 [B]; all CUDA tensors.
+    Returns (o [B,Hq,D] bf16, lse [B,Hq] fp32).  The fp32 workspace for the
+    split partials is allocated here unless one is passed."""
+    import torch
+    for name, t in (("q", q), ("k_cache", k_cache), ("v_cache", v_cache)):
+        if not t.is_cuda or t.dtype != torch.bfloat16 or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous bf16 CUDA tensor")
+    for name, t in (("page_table", page_table), ("seq_lens", seq_lens)):
+        if not t.is_cuda or t.dtype != torch.int32 or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous int32 CUDA tensor")
+    if q.dim() != 3 or k_cache.dim() != 4 or k_cache.shape != v_cache.shape:
+        raise ValueError("q [B,Hq,D], k_cache/v_cache [num_pages, page_size, Hkv, D]")
+    B, Hq, D = q.shape
+    num_pages, page_size, Hkv, Dk = k_cache.shape
+    if Dk != D or page_table.dim() != 2 or page_table.shape[0] != B or seq_lens.shape != (B,):
+        raise ValueError("shapes do not match")
+    max_pages = page_table.shape[1]
+    if scale is None:
+        scale = 1.0 / float(D) ** 0.5
+    if out is None:
+        out = torch.empty_like(q)
+    if lse is None:
+        lse = torch.empty((B, Hq), dtype=torch.float32, device=q.device)
+    need = mk_attn_decode_workspace_bytes(B, Hq, Hkv, D, page_size, max_pages)
+    if need < 0:
+        raise MkAttnError(MK_ERR_INVALID_ARG, "invalid decode sizes")
+    if workspace is None and need > 0:
+        workspace = torch.empty((need + 15) // 16 * 4, dtype=torch.float32, device=q.device)
+    ws_ptr = None if workspace is None else workspace.data_ptr()
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    if stream is None:
+        stream = torch.cuda.current_stream(q.device)
+    _check(mk_attn_decode_paged(q.data_ptr(), k_cache.data_ptr(), v_cache.data_ptr(),
+                                page_table.data_ptr(), seq_lens.data_ptr(), out.data_ptr(),
+                                lse.data_ptr(), B, Hq, Hkv, D, page_size, max_pages, num_pages,
+                                float(scale), ws_ptr, ws_bytes, stream.cuda_stream))
     return out, lse

@@ -52,6 +52,7 @@
 
 #include "mk_attn.h"
 #include "ptx.cuh"
+#include "tma_host.h"
 
 namespace mk {
 
@@ -813,34 +814,6 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // =================================================================== host
 
-static PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void *ptr = nullptr;
-    cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
-                                         cudaEnableDefault, &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-  });
-  return fn;
-}
-
-// [tokens, heads, D] bf16, boxes of 128 tokens x 1 head x 64 elements, 128-byte swizzle.
-static bool encode_tokens_heads_dim(CUtensorMap *map, const void *base, uint64_t tokens,
-                                    uint64_t heads, uint64_t D) {
-  auto enc = tensor_map_encoder();
-  if (!enc) return false;
-  const cuuint64_t dims[3] = {D, heads, tokens};
-  const cuuint64_t strides[2] = {D * 2, heads * D * 2};
-  const cuuint32_t box[3] = {(cuuint32_t)kBoxCols, 1, (cuuint32_t)kTile};
-  const cuuint32_t estr[3] = {1, 1, 1};
-  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides,
-             box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 struct DeviceInfo {
   std::once_flag once;
   int sm_count = 0;
@@ -867,9 +840,9 @@ static int launch(const void *q, const void *k, const void *v, const Params &p, 
                   cudaStream_t stream) {
   using C = KernelCfg<D>;
   CUtensorMap tq, tk, tv;
-  if (!encode_tokens_heads_dim(&tq, q, tokens, p.Hq, D) ||
-      !encode_tokens_heads_dim(&tk, k, tokens, p.Hkv, D) ||
-      !encode_tokens_heads_dim(&tv, v, tokens, p.Hkv, D))
+  if (!encode_tokens_heads_dim(&tq, q, tokens, p.Hq, D, kTile) ||
+      !encode_tokens_heads_dim(&tk, k, tokens, p.Hkv, D, kTile) ||
+      !encode_tokens_heads_dim(&tv, v, tokens, p.Hkv, D, kTile))
     return MK_ERR_CUDA;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return MK_ERR_CUDA;
@@ -977,9 +950,9 @@ int mk_attn_check_status(void *stream) {
   if (h != 0) {
     const int zero = 0;
     if (cudaMemcpyToSymbol(mk::g_status, &zero, sizeof(int)) != cudaSuccess) return MK_ERR_CUDA;
-    return h;
   }
-  return MK_OK;
+  const int hd = mk::decode_take_status();
+  return h != 0 ? h : hd;
 }
 
 int mk_attn_version(void) { return 300; }
