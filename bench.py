@@ -13,8 +13,13 @@ on its own GPU (weak scaling: the work units of attention -- sequence, head,
 query tile -- are independent, so there is no data-path collective); ranks
 meet at a barrier around the timed region and rank 0 reports the maximum time.
 
+--workload decode instead times one paged decode step (mk_attn_decode_paged:
+64 sequences of 1024-8192 cached tokens, Hq=32, Hkv=8, D=128, page_size=64)
+and reports HBM GB/s against the measured copy bandwidth.
+
 --impl reference times the fp64 CPU oracle on bounded row samples of the same
-workload (rank 0 only; other ranks exit without work).
+workload (the whole step for decode; rank 0 only; other ranks exit without
+work).
 """
 from __future__ import annotations
 
@@ -32,9 +37,11 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "attention fwd TFLOP/s (causal FLOPs) and % of GB300 bf16 tensor peak"
+DECODE_METRIC = "paged decode step HBM GB/s (algorithmic bytes) and % of measured HBM copy bandwidth"
 NOMINAL_BF16_TFLOPS = 2250.0
 FLUSH_BYTES = 256 << 20
 KERNEL_SOURCES = ["paper_2609_04523_gb300/csrc/fmha_fwd.cu", "paper_2609_04523_gb300/csrc/ptx.cuh"]
+DECODE_SOURCES = ["paper_2609_04523_gb300/csrc/decode.cu", "paper_2609_04523_gb300/csrc/ptx.cuh"]
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "ncu_traffic.json")
 BAD_REASONS = {"hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown"}
 
@@ -45,6 +52,9 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5])
+    ap.add_argument("--workload", default="prefill", choices=["prefill", "decode"],
+                    help="prefill: the attention forward pass (--config); decode: one paged "
+                         "decode step (the decode workload below)")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
@@ -62,15 +72,15 @@ def measured_peaks():
         return {"bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "hbm_gbs": 6800.0}, "fallback"
 
 
-def kernel_source_hash() -> str:
+def kernel_source_hash(sources=KERNEL_SOURCES) -> str:
     h = hashlib.sha256()
-    for rel in KERNEL_SOURCES:
+    for rel in sources:
         with open(os.path.join(ROOT, rel), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
 
 
-def ncu_traffic(workload: str):
+def ncu_traffic(workload: str, sources=KERNEL_SOURCES):
     """DRAM bytes per launch from a committed ncu summary, or None when there is
     none for this workload or the kernel source changed since it was taken."""
     try:
@@ -78,7 +88,7 @@ def ncu_traffic(workload: str):
             rec = json.load(f).get(workload)
     except (OSError, ValueError):
         return None
-    if not rec or rec.get("kernel_source_hash") != kernel_source_hash():
+    if not rec or rec.get("kernel_source_hash") != kernel_source_hash(sources):
         return None
     return rec.get("dram_bytes_per_launch")
 
@@ -429,6 +439,220 @@ def run_ours(args, rank: int, world: int, local_rank: int):
     return line
 
 
+# ----------------------------------------------------------- decode step
+
+DECODE_NAME = "decode_gqa_b64_hq32_hkv8_d128_ps64_ctx1k-8k"
+DECODE_DESC = ("one paged decode step, B=64 sequences, Hq=32, Hkv=8, D=128, page_size=64, "
+               "context lengths uniform in [1024, 8192] by seed, pages in random order")
+
+
+def decode_inputs():
+    import numpy as np
+    from paper_2609_04523_gb300 import workloads as W
+    lens = [int(x) for x in np.random.default_rng(2001).integers(1024, 8193, size=64)]
+    return W.make_paged(lens, 32, 8, 128, 64, seed=2001, spare_pages=64)
+
+
+def cpu_oracle_decode(inp):
+    """The oracle, as it stands, on the whole decode step (a few GFLOP)."""
+    import oracle
+    t0 = time.perf_counter()
+    o, lse = oracle.decode_paged(inp.q, inp.k_cache, inp.v_cache, inp.page_table, inp.seq_lens,
+                                 inp.scale)
+    return time.perf_counter() - t0, oracle.default_threads(), o, lse
+
+
+def run_decode(args, rank: int, world: int, local_rank: int):
+    import numpy as np
+    import torch
+
+    from paper_2609_04523_gb300 import decode_paged, mk_attn_check_status
+    from paper_2609_04523_gb300 import workloads as W
+    from paper_2609_04523_gb300.build import build_library
+
+    build_library()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    inp = decode_inputs()
+    lens = [int(x) for x in inp.seq_lens]
+    B, Hq, D = inp.q.shape
+    Hkv = inp.k_cache.shape[2]
+    nbytes = W.decode_bytes(lens, Hq, Hkv, D)
+    q, kc, vc, pt, sl = (t.to(dev) for t in (inp.q, inp.k_cache, inp.v_cache, inp.page_table,
+                                             inp.seq_lens))
+    o = torch.empty_like(q)
+    lse = torch.empty((B, Hq), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    props = torch.cuda.get_device_properties(dev)
+    pci_bus_id = None
+    if hasattr(props, "pci_bus_id"):
+        pci_bus_id = "%08x:%02x:%02x.0" % (getattr(props, "pci_domain_id", 0), props.pci_bus_id,
+                                           getattr(props, "pci_device_id", 0))
+    from paper_2609_04523_gb300 import mk_attn_decode_workspace_bytes
+    need = mk_attn_decode_workspace_bytes(B, Hq, Hkv, D, inp.k_cache.shape[1], pt.shape[1])
+    ws = torch.empty(max(need, 16) // 4, dtype=torch.float32, device=dev) if need > 0 else None
+    launches = 2 if need > 0 else 1
+
+    def step():
+        decode_paged(q, kc, vc, pt, sl, inp.scale, out=o, lse=lse, workspace=ws, stream=stream)
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize(dev)
+    if mk_attn_check_status(stream.cuda_stream) != 0:
+        raise RuntimeError("decode kernel reported an error during warm-up")
+
+    def timed_region():
+        starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize(dev)
+        with ClockSampler(pci_bus_id, local_rank) as cs:
+            for i in range(args.steps):
+                flush.zero_()
+                starts[i].record(stream)
+                step()
+                ends[i].record(stream)
+            torch.cuda.synchronize(dev)
+        if world > 1:
+            torch.distributed.barrier()
+        return [a.elapsed_time(b) for a, b in zip(starts, ends)], cs.summary()
+
+    ms, clocks = timed_region()
+    remeasured = False
+    if clocks_rejected(clocks):
+        ms, clocks = timed_region()
+        remeasured = True
+    if mk_attn_check_status(stream.cuda_stream) != 0:
+        raise RuntimeError("decode kernel reported an error in the timed region")
+    total_ms = max_over_ranks(sum(ms), world, dev)
+    ms_per_step = total_ms / args.steps
+    gbs_job = world * nbytes * args.steps / (total_ms * 1e-3) / 1e9
+    gbs = nbytes / (ms_per_step * 1e-3) / 1e9
+
+    # End to end: the cache stays on the device (it is the server's state);
+    # each step copies the new queries, page table and lengths in and o, lse out.
+    qh, pth, slh = inp.q.pin_memory(), inp.page_table.pin_memory(), inp.seq_lens.pin_memory()
+    oh = torch.empty(o.shape, dtype=o.dtype).pin_memory()
+    lh = torch.empty(lse.shape, dtype=lse.dtype).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for t in (qh, pth, slh))
+    d2h = oh.numel() * oh.element_size() + lh.numel() * lh.element_size()
+    qd, ptd, sld = torch.empty_like(q), torch.empty_like(pt), torch.empty_like(sl)
+
+    def e2e_step():
+        qd.copy_(qh, non_blocking=True)
+        ptd.copy_(pth, non_blocking=True)
+        sld.copy_(slh, non_blocking=True)
+        decode_paged(qd, kc, vc, ptd, sld, inp.scale, out=o, lse=lse, workspace=ws, stream=stream)
+        oh.copy_(o, non_blocking=True)
+        lh.copy_(lse, non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        torch.distributed.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    e2e_gbs = world * nbytes * args.steps / (e2e_ms * 1e-3) / 1e9
+
+    if rank != 0:
+        return None
+    peaks, peak_src = measured_peaks()
+    peak = float(peaks["hbm_gbs"])
+    line = {
+        "metric": DECODE_METRIC,
+        "value": round(gbs_job, 1),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 5),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) bf16 query and cache, seeded lengths and page order)",
+        "config": {
+            "workload": f"{DECODE_NAME}: {DECODE_DESC}",
+            "bytes_per_step_per_gpu": nbytes,
+            "byte_convention": "every cached key and value read once, q read, o and lse written",
+            "cached_keys": sum(lens),
+            "l2": "flushed before every timed step (256 MiB device write, outside the event pair); "
+                  "the cache (%.2f GB) is far larger than L2" % (4 * sum(lens) * Hkv * D / 1e9),
+            "timing": "CUDA events around each call (decode kernel and, with several KV splits, "
+                      "the merge kernel) on the launching stream; sum over steps",
+            "parallelism": f"replicas x{world} (independent workloads per GPU)",
+        },
+        "roofline": {
+            "bound": "hbm",
+            "achieved": round(gbs, 1),
+            "peak": peak,
+            "unit": "GB/s",
+            "frac": round(gbs / peak, 4),
+            "traffic": ncu_traffic(DECODE_NAME, DECODE_SOURCES),
+            "peak_source": f"{peak_src} HBM copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
+            "kernel": "mk::dec::decode_kernel<128, 4>" + (" + merge_kernel<128>" if need > 0 else ""),
+        },
+        "e2e": {"value": round(e2e_gbs, 1), "unit": "GB/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": args.steps * launches,
+        "clocks": clocks,
+    }
+    if remeasured:
+        line["clocks_note"] = "first timed region saw a rejected clock state; re-measured once"
+    if not args.no_cpu_baseline:
+        secs, cores, o_ref, lse_ref = cpu_oracle_decode(inp)
+        line["cpu_baseline"] = {"value": round(nbytes / secs / 1e9, 3), "unit": "GB/s",
+                                "cores": cores, "kind": "oracle",
+                                "sample": f"the whole decode step, {secs:.1f} s on {cores} threads"}
+        d = o.float().cpu().double().numpy() - o_ref
+        line["parity_spot_check"] = {
+            "rows": int(B * Hq),
+            "o_max_abs": float(np.max(np.abs(d))),
+            "o_rel_rms": float(math.sqrt(np.sum(d * d) / np.sum(o_ref * o_ref))),
+            "lse_max_abs": float(np.max(np.abs(lse.double().cpu().numpy() - lse_ref))),
+        }
+    return line
+
+
+def run_decode_reference(args, rank: int):
+    """The oracle, as it stands, timed on the whole decode step per step."""
+    if rank != 0:
+        return None
+    inp = decode_inputs()
+    lens = [int(x) for x in inp.seq_lens]
+    from paper_2609_04523_gb300 import workloads as W
+    nbytes = W.decode_bytes(lens, inp.q.shape[1], inp.k_cache.shape[2], inp.q.shape[2])
+    vals, cores, secs = [], None, 0.0
+    for i in range(args.warmup + args.steps):
+        secs, cores, _, _ = cpu_oracle_decode(inp)
+        if i >= args.warmup:
+            vals.append(nbytes / secs / 1e9)
+    value = statistics.median(vals)
+    return {
+        "impl": "reference", "metric": DECODE_METRIC, "value": round(value, 3), "unit": "GB/s",
+        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": None,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded N(0,1) bf16 query and cache, seeded lengths and page order)",
+        "config": {"workload": f"{DECODE_NAME}: {DECODE_DESC}",
+                   "note": "the fp64 CPU oracle, as it stands, on the whole step"},
+        "cpu_baseline": {"value": round(value, 3), "unit": "GB/s", "cores": cores, "kind": "oracle",
+                         "sample": f"per step: the whole decode step, {secs:.1f} s"},
+        "e2e": {"value": round(value, 3), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+        "gpu_launches": 0,
+    }
+
+
 # ----------------------------------------------------------- reference arm
 
 def run_reference(args, rank: int):
@@ -477,7 +701,8 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
-        line = run_reference(args, rank)
+        line = run_decode_reference(args, rank) if args.workload == "decode" else \
+            run_reference(args, rank)
         if line is not None:
             print(json.dumps(line), flush=True)
         return
@@ -486,7 +711,8 @@ def main():
         torch.cuda.set_device(local_rank)
         torch.distributed.init_process_group("nccl")
     try:
-        line = run_ours(args, rank, world, local_rank)
+        line = run_decode(args, rank, world, local_rank) if args.workload == "decode" else \
+            run_ours(args, rank, world, local_rank)
     finally:
         if world > 1:
             import torch

@@ -129,7 +129,8 @@ MK_API int64_t mk_attn_decode_workspace_bytes(int B, int Hq, int Hkv, int D, int
  *   lse          fp32 [B, Hq] output, fully overwritten (natural log, scale
  *                included); L_b = 0 gives o = 0 and lse = -inf.
  *   D            64 or 128.   page_size  16, 32, 64 or 128.
- *   Hq / Hkv     at most 16.
+ *   Hq / Hkv     any; Hkv * ceil(Hq / Hkv / 8) at most 65535, B at most
+ *                65535.
  *   workspace    device buffer of at least mk_attn_decode_workspace_bytes()
  *                bytes, 16-byte aligned, or NULL when that is 0.  Scratch
  *                for the per-split partial results; its contents on entry
@@ -138,7 +139,7 @@ MK_API int64_t mk_attn_decode_workspace_bytes(int B, int Hq, int Hkv, int D, int
  *   stream       cudaStream_t; the call is asynchronous and never syncs.
  * Returns MK_OK; MK_ERR_INVALID_ARG (null pointer, sizes out of range, a
  * missing or too small workspace), MK_ERR_UNSUPPORTED (D, page_size, or a
- * head group above 16), MK_ERR_ALIGNMENT (q, caches, o or workspace not
+ * grid beyond those limits), MK_ERR_ALIGNMENT (q, caches, o or workspace not
  * 16-byte aligned; page_table, seq_lens or lse not 4-byte aligned), or
  * MK_ERR_CUDA.  On any error nothing is launched.  Page-table entries or
  * lengths out of range, which only the device sees, leave o and lse undefined

@@ -48,12 +48,20 @@ def check(inp, what):
 
 @pytest.mark.parametrize("D", [64, 128])
 @pytest.mark.parametrize("page_size", [16, 32, 64, 128])
-@pytest.mark.parametrize("G", [1, 4, 8])
+@pytest.mark.parametrize("G", [1, 2, 3, 4, 8, 11, 16])
 def test_decode_lengths(D, page_size, G):
+    """G picks the CTA's head capacity (1, 2, 4, 8); 3 leaves capacity unused,
+    11 splits a group into CTAs of 6 and 5 heads, 16 into two full CTAs."""
     lens = [0, 1, page_size - 1, page_size, page_size + 1, 3 * page_size + 7, 1000, 2049]
     Hkv = 2
     inp = W.make_paged(lens, Hkv * G, Hkv, D, page_size, seed=600 + D + page_size + G)
     check(inp, f"D{D} ps{page_size} G{G}")
+
+
+def test_decode_wide_group():
+    """32 query heads per key/value head: four CTAs of 8 heads each."""
+    inp = W.make_paged([1, 700, 2500], 64, 2, 128, 32, seed=655)
+    check(inp, "G32")
 
 
 @pytest.mark.parametrize("B", [1, 3, 40])
