@@ -40,7 +40,9 @@ typedef enum {
     MK_ERR_UNSUPPORTED = -2,  /* head dimension other than 64 or 128 */
     MK_ERR_ALIGNMENT = -3,    /* a base pointer not 16-byte aligned */
     MK_ERR_CUDA = -4,         /* a CUDA runtime/driver call failed */
-    MK_ERR_TIMEOUT = -5       /* a kernel wait ran out; reported by mk_attn_check_status */
+    MK_ERR_TIMEOUT = -5,      /* a kernel wait ran out; reported by mk_attn_check_status */
+    MK_ERR_SCRATCH_LIMIT = -6 /* sizes need more than MK_ATTN_DECODE_STATIC_SCRATCH_BYTES of
+                                 scratch (mk_attn_decode_paged_noalloc only) */
 } mk_status;
 
 /*
@@ -150,6 +152,42 @@ MK_API int mk_attn_decode_paged(const void *q, const void *k_cache, const void *
                                 float *lse, int B, int Hq, int Hkv, int D, int page_size,
                                 int max_pages, int num_pages, float scale, void *workspace,
                                 int64_t workspace_bytes, void *stream);
+
+/* Size of the library's own decode scratch array (8 MiB), which every GPU
+ * that loads the library holds until the process exits. */
+#define MK_ATTN_DECODE_STATIC_SCRATCH_BYTES (8 * 1024 * 1024)
+
+/*
+ * mk_attn_decode_paged_noalloc -- mk_attn_decode_paged for callers that
+ * cannot allocate device memory: code that runs where cudaMalloc is not
+ * allowed or not wanted (inside a host callback, under an allocator that
+ * another runtime owns, or in a plugin that must not touch the device heap).
+ * The paper has no counterpart; it is an addition of this library.
+ *
+ * Arguments, layouts, results and errors are those of mk_attn_decode_paged
+ * without `workspace` and `workspace_bytes`: the per-split partial results
+ * go to a scratch array of MK_ATTN_DECODE_STATIC_SCRATCH_BYTES bytes that
+ * the library declares in device memory (one per GPU).  The call allocates
+ * nothing and calls no allocating routine.
+ *
+ *   - Sizes for which mk_attn_decode_workspace_bytes() exceeds
+ *     MK_ATTN_DECODE_STATIC_SCRATCH_BYTES return MK_ERR_SCRATCH_LIMIT and
+ *     launch nothing; use mk_attn_decode_paged with a workspace for those.
+ *   - The first call on each device looks up that device's address of the
+ *     array (with the device current) and keeps it; make that first call
+ *     before any stream capture on the device.  A failed lookup returns
+ *     MK_ERR_CUDA.
+ *   - Every call on a device shares the one array, which keeps whatever the
+ *     last call left there (nothing in it needs to start at zero: each call
+ *     writes every partial it reads).  Calls whose kernels can overlap on the
+ *     GPU -- on different streams with no ordering between them, or from
+ *     several host threads -- race on it; order them (one stream, or events).
+ */
+MK_API int mk_attn_decode_paged_noalloc(const void *q, const void *k_cache, const void *v_cache,
+                                        const int32_t *page_table, const int32_t *seq_lens,
+                                        void *o, float *lse, int B, int Hq, int Hkv, int D,
+                                        int page_size, int max_pages, int num_pages, float scale,
+                                        void *stream);
 
 /* Short static description of a status code.  Never NULL. */
 MK_API const char *mk_attn_error_string(int status);

@@ -19,11 +19,15 @@ MK_ERR_UNSUPPORTED = -2
 MK_ERR_ALIGNMENT = -3
 MK_ERR_CUDA = -4
 MK_ERR_TIMEOUT = -5
+MK_ERR_SCRATCH_LIMIT = -6
+
+# Bytes of the library's own decode scratch array (MK_ATTN_DECODE_STATIC_SCRATCH_BYTES).
+DECODE_STATIC_SCRATCH_BYTES = 8 * 1024 * 1024
 
 # Symbols declared in include/mk_attn.h.
 EXPORTED = ("mk_attn_fwd", "mk_attn_fwd_stall_test", "mk_attn_decode_workspace_bytes",
-            "mk_attn_decode_paged", "mk_attn_error_string", "mk_attn_check_status",
-            "mk_attn_version")
+            "mk_attn_decode_paged", "mk_attn_decode_paged_noalloc", "mk_attn_error_string",
+            "mk_attn_check_status", "mk_attn_version")
 
 _lock = threading.Lock()
 _lib = None
@@ -61,6 +65,9 @@ def load_library() -> ctypes.CDLL:
             lib.mk_attn_decode_paged.argtypes = [vp, vp, vp, vp, vp, vp, vp, i, i, i, i, i, i, i,
                                                  ctypes.c_float, vp, i64, vp]
             lib.mk_attn_decode_paged.restype = i
+            lib.mk_attn_decode_paged_noalloc.argtypes = [vp, vp, vp, vp, vp, vp, vp, i, i, i, i, i,
+                                                         i, i, ctypes.c_float, vp]
+            lib.mk_attn_decode_paged_noalloc.restype = i
             lib.mk_attn_error_string.argtypes = [i]
             lib.mk_attn_error_string.restype = ctypes.c_char_p
             lib.mk_attn_check_status.argtypes = [vp]
@@ -167,6 +174,18 @@ def mk_attn_decode_paged(q: int, k_cache: int, v_cache: int, page_table: int, se
                                                B, Hq, Hkv, D, page_size, max_pages, num_pages,
                                                float(scale), workspace, int(workspace_bytes),
                                                stream)
+
+
+def mk_attn_decode_paged_noalloc(q: int, k_cache: int, v_cache: int, page_table: int,
+                                 seq_lens: int, o: int, lse: int, B: int, Hq: int, Hkv: int,
+                                 D: int, page_size: int, max_pages: int, num_pages: int,
+                                 scale: float, stream: int | None) -> int:
+    """Raw C-ABI call of the decode step that uses the library's static
+    scratch instead of a caller workspace: integer device pointers in, status
+    code out."""
+    return load_library().mk_attn_decode_paged_noalloc(q, k_cache, v_cache, page_table, seq_lens,
+                                                       o, lse, B, Hq, Hkv, D, page_size,
+                                                       max_pages, num_pages, float(scale), stream)
 
 
 def decode_paged(q, k_cache, v_cache, page_table, seq_lens, scale: float | None = None,

@@ -41,6 +41,7 @@
 
 #include <cmath>
 #include <cstdint>
+#include <mutex>
 
 #include "mk_attn.h"
 #include "ptx.cuh"
@@ -530,6 +531,37 @@ static int launch(const CUtensorMap &tk, const CUtensorMap &tv, const Params &p,
   return MK_OK;
 }
 
+// Scratch of mk_attn_decode_paged_noalloc: the split partials of every call
+// on this device, for callers that cannot allocate device memory.  Host code
+// sees only a stand-in for it; its device address is looked up once per
+// device (with that device current) and then passed to the kernels like a
+// caller's workspace.
+constexpr int64_t kStaticScratchBytes = MK_ATTN_DECODE_STATIC_SCRATCH_BYTES;
+static __device__ __align__(256) float g_static_scratch[kStaticScratchBytes / sizeof(float)];
+
+struct StaticScratch {
+  std::mutex mu;
+  void *addr[64] = {};
+};
+static StaticScratch g_scratch;
+
+// Device address of g_static_scratch on the current device, or nullptr if
+// the lookup fails (then retried on the next call).
+static void *static_scratch_address() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lock(g_scratch.mu);
+  if (!g_scratch.addr[dev]) {
+    void *ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_static_scratch) != cudaSuccess || !ptr) {
+      cudaGetLastError();  // not sticky: leave no error behind for the caller
+      return nullptr;
+    }
+    g_scratch.addr[dev] = ptr;
+  }
+  return g_scratch.addr[dev];
+}
+
 }  // namespace dec
 
 int decode_take_status() {
@@ -627,6 +659,23 @@ int mk_attn_decode_paged(const void *q, const void *k_cache, const void *v_cache
   if (HG == 2) return dec::launch<64, 2>(tk, tv, p, st);
   if (HG <= 4) return dec::launch<64, 4>(tk, tv, p, st);
   return dec::launch<64, dec::kMaxHeads>(tk, tv, p, st);
+}
+
+
+int mk_attn_decode_paged_noalloc(const void *q, const void *k_cache, const void *v_cache,
+                                 const int32_t *page_table, const int32_t *seq_lens, void *o,
+                                 float *lse, int B, int Hq, int Hkv, int D, int page_size,
+                                 int max_pages, int num_pages, float scale, void *stream) {
+  // Set-up on the first call per device, whether or not these sizes need
+  // scratch, so that the lookup never happens later during a stream capture.
+  void *scratch = mk::dec::static_scratch_address();
+  if (!scratch) return MK_ERR_CUDA;
+  const int64_t need = mk_attn_decode_workspace_bytes(B, Hq, Hkv, D, page_size, max_pages);
+  if (need > mk::dec::kStaticScratchBytes) return MK_ERR_SCRATCH_LIMIT;
+  // Invalid sizes (need < 0) are reported by the checks of mk_attn_decode_paged.
+  return mk_attn_decode_paged(q, k_cache, v_cache, page_table, seq_lens, o, lse, B, Hq, Hkv, D,
+                              page_size, max_pages, num_pages, scale, scratch,
+                              mk::dec::kStaticScratchBytes, stream);
 }
 
 }  // extern "C"

@@ -938,6 +938,7 @@ const char *mk_attn_error_string(int status) {
     case MK_ERR_ALIGNMENT: return "pointer not 16-byte aligned";
     case MK_ERR_CUDA: return "CUDA call failed";
     case MK_ERR_TIMEOUT: return "kernel wait timed out";
+    case MK_ERR_SCRATCH_LIMIT: return "sizes need more scratch than the static decode array holds";
     default: return "unknown status";
   }
 }
