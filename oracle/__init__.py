@@ -1,4 +1,5 @@
-"""fp64 CPU oracle for the attention forward pass (TEST INFRASTRUCTURE).
+"""fp64 CPU oracle for the attention forward and backward passes and the paged
+decode step (TEST INFRASTRUCTURE).
 
 Only ``tests/``, ``__graft_entry__.smoke()`` and ``bench.py``'s cpu_baseline /
 reference legs may import this package.  The product path never does, and the
@@ -66,6 +67,16 @@ def _bind(lib: ctypes.CDLL) -> ctypes.CDLL:
     lib.mk_oracle_decode_paged_f64.argtypes = [p, p, p, p, p, p, p, i, i, i, i, i, i, i,
                                                ctypes.c_double, i]
     lib.mk_oracle_decode_paged_f64.restype = i
+    lib.mk_oracle_attn_bwd_f64.argtypes = [p, p, p, p, p, p, p, i, i, i, i, i, i,
+                                           ctypes.c_double, p, i]
+    lib.mk_oracle_attn_bwd_f64.restype = i
+    lib.mk_oracle_attn_bwd_dq_rows_f64.argtypes = [p, p, p, p, i, i, i, i, i, i, ctypes.c_double,
+                                                   p, p, ctypes.c_int64, p, i]
+    lib.mk_oracle_attn_bwd_dq_rows_f64.restype = i
+    lib.mk_oracle_attn_bwd_dkv_ranges_f64.argtypes = [p, p, p, p, i, i, i, i, i, i,
+                                                      ctypes.c_double, p, p, ctypes.c_int64, p,
+                                                      p, i]
+    lib.mk_oracle_attn_bwd_dkv_ranges_f64.restype = i
     return lib
 
 
@@ -187,3 +198,66 @@ def decode_paged(q, k_cache, v_cache, page_table, seq_lens, scale: float,
     if st != 0:
         raise ValueError(f"oracle rejected the decode problem (status {st})")
     return o, lse
+
+
+def attn_bwd(q, k, v, do, causal: bool, scale: float, cu_seqlens=None,
+             n_threads: int | None = None, lib: ctypes.CDLL | None = None):
+    """Full backward pass in fp64: the gradients of the forward definition
+    with respect to q, k and v for the output gradient `do` (layout of q).
+
+    Returns (dq, dk, dv) as fp64 numpy arrays shaped like q, k, v."""
+    qb, kb, vb, dob = _bits(q), _bits(k), _bits(v), _bits(do)
+    if dob.shape != qb.shape:
+        raise ValueError("do must have the shape of q")
+    cu = _cu(cu_seqlens)
+    B, Hq, Hkv, S, D = _shape(qb, kb, cu)
+    dq = np.zeros(qb.shape, dtype=np.float64)
+    dk = np.zeros(kb.shape, dtype=np.float64)
+    dv = np.zeros(vb.shape, dtype=np.float64)
+    lib = lib or load()
+    st = lib.mk_oracle_attn_bwd_f64(_ptr(qb), _ptr(kb), _ptr(vb), _ptr(dob), _ptr(dq), _ptr(dk),
+                                    _ptr(dv), B, Hq, Hkv, S, D, int(bool(causal)), float(scale),
+                                    _ptr(cu), int(n_threads or default_threads()))
+    if st != 0:
+        raise ValueError(f"oracle rejected the problem (status {st})")
+    return dq, dk, dv
+
+
+def attn_bwd_dq_rows(q, k, v, do, causal: bool, scale: float, rows, cu_seqlens=None,
+                     n_threads: int | None = None, lib: ctypes.CDLL | None = None):
+    """dq of the backward pass on selected rows (b, h, i) only: [n, D] fp64."""
+    qb, kb, vb, dob = _bits(q), _bits(k), _bits(v), _bits(do)
+    cu = _cu(cu_seqlens)
+    B, Hq, Hkv, S, D = _shape(qb, kb, cu)
+    r = np.ascontiguousarray(np.asarray(rows, dtype=np.int64).reshape(-1, 3))
+    out = np.zeros((r.shape[0], D), dtype=np.float64)
+    lib = lib or load()
+    st = lib.mk_oracle_attn_bwd_dq_rows_f64(_ptr(qb), _ptr(kb), _ptr(vb), _ptr(dob), B, Hq, Hkv,
+                                            S, D, int(bool(causal)), float(scale), _ptr(cu),
+                                            _ptr(r), r.shape[0], _ptr(out),
+                                            int(n_threads or default_threads()))
+    if st != 0:
+        raise ValueError(f"oracle rejected the rows (status {st})")
+    return out
+
+
+def attn_bwd_dkv_ranges(q, k, v, do, causal: bool, scale: float, ranges, cu_seqlens=None,
+                        n_threads: int | None = None, lib: ctypes.CDLL | None = None):
+    """dk and dv of the backward pass for key ranges (b, g, j0, j1) of a
+    sequence and key/value head (positions within the sequence).  Returns
+    (dk_rows, dv_rows), each [sum of (j1 - j0), D] fp64, ranges in order."""
+    qb, kb, vb, dob = _bits(q), _bits(k), _bits(v), _bits(do)
+    cu = _cu(cu_seqlens)
+    B, Hq, Hkv, S, D = _shape(qb, kb, cu)
+    r = np.ascontiguousarray(np.asarray(ranges, dtype=np.int64).reshape(-1, 4))
+    n = int(np.sum(r[:, 3] - r[:, 2])) if r.size else 0
+    dk = np.zeros((max(n, 0), D), dtype=np.float64)
+    dv = np.zeros((max(n, 0), D), dtype=np.float64)
+    lib = lib or load()
+    st = lib.mk_oracle_attn_bwd_dkv_ranges_f64(_ptr(qb), _ptr(kb), _ptr(vb), _ptr(dob), B, Hq,
+                                               Hkv, S, D, int(bool(causal)), float(scale),
+                                               _ptr(cu), _ptr(r), r.shape[0], _ptr(dk), _ptr(dv),
+                                               int(n_threads or default_threads()))
+    if st != 0:
+        raise ValueError(f"oracle rejected the ranges (status {st})")
+    return dk, dv

@@ -1,5 +1,6 @@
 /*
- * mk_oracle.c -- plain fp64 CPU oracle for the attention forward pass.
+ * mk_oracle.c -- plain fp64 CPU oracle for the attention forward pass, its
+ * backward pass (gradients of q, k, v) and one paged decode step.
  *
  * TEST INFRASTRUCTURE.  Only tests/, __graft_entry__.smoke() and bench.py's
  * cpu_baseline / reference legs may load this file's library.  The product
@@ -415,4 +416,344 @@ int mk_oracle_decode_paged_f64(const uint16_t *q, const uint16_t *k_cache,
     decode_job_t job = {q, k_cache, v_cache, page_table, seq_lens, o, lse, B, Hq, Hkv, D,
                         page_size, max_pages, scale, &next, max_len};
     return run_threads(decode_worker, &job, sizeof job, n_threads);
+}
+
+/* ------------------------------------------------------------ backward pass */
+
+/*
+ * Gradients of the forward definition with respect to q, k and v, given dO,
+ * the gradient of a loss with respect to o (the training step's backward
+ * pass of the same reference operation).  Reverse-mode chain rule through
+ * the definition, written out for every sequence b, key/value head g, query
+ * head h of g's group and query position i:
+ *
+ *   P_ij    = exp(s_ij - lse_i)                       j in K_i (0 elsewhere)
+ *   dP_ij   = sum_d dO[i,h,d] * v[j,g,d]              (dL/dP_ij, since o_i = sum_j P_ij v_j)
+ *   Delta_i = sum_{j in K_i} P_ij * dP_ij
+ *   dS_ij   = P_ij * (dP_ij - Delta_i)                (dL/ds_ij through the softmax)
+ *   dq[i,h] = scale * sum_{j in K_i} dS_ij * k[j,g]   (s_ij = scale * q_i . k_j)
+ *   dk[j,g] = scale * sum_{h in group g} sum_{i : j in K_i} dS_ij * q[i,h]
+ *   dv[j,g] =         sum_{h in group g} sum_{i : j in K_i} P_ij * dO[i,h]
+ *
+ * s_ij and lse_i are recomputed here in fp64 from the bf16 inputs (the
+ * forward definition above), and Delta_i is the sum over P_ij dP_ij itself,
+ * not a product with a rounded o.  dq has the layout of q, dk and dv that of
+ * k and v; dO that of q.  A key that no query sees gets dk = dv = 0.
+ */
+typedef struct {
+    const problem_t *p;
+    const uint16_t *dO;
+    double *dq, *dk, *dv;
+    int64_t n_tasks; /* (b, g) pairs */
+    int64_t *next;
+    int max_len;
+} bwd_job_t;
+
+/* Row statistics of (b, h, i): s_buf[j] = s_ij for j < n_keys, returns lse_i
+ * (-inf for an empty row). */
+static double row_scores(const problem_t *p, int64_t tok0, int g, int h, int i, int n_keys,
+                         double *s_buf)
+{
+    const int D = p->D;
+    const uint16_t *qi = p->q + ((tok0 + i) * p->Hq + h) * (int64_t)D;
+    double m = -INFINITY;
+    for (int j = 0; j < n_keys; ++j) {
+        const uint16_t *kj = p->k + ((tok0 + j) * p->Hkv + g) * (int64_t)D;
+        double dot = 0.0;
+        for (int d = 0; d < D; ++d)
+            dot += bf16_bits_to_f64(qi[d]) * bf16_bits_to_f64(kj[d]);
+        s_buf[j] = p->scale * dot;
+        if (s_buf[j] > m)
+            m = s_buf[j];
+    }
+    if (n_keys == 0)
+        return -INFINITY;
+    double l = 0.0;
+    for (int j = 0; j < n_keys; ++j)
+        l += exp(s_buf[j] - m);
+    return m + log(l);
+}
+
+/* P_ij into s_buf and dP_ij into dp_buf for j < n_keys; returns Delta_i. */
+static double row_probs(const problem_t *p, const uint16_t *dO, int64_t tok0, int g, int h,
+                        int i, int n_keys, double *s_buf, double *dp_buf)
+{
+    const int D = p->D;
+    const double lse = row_scores(p, tok0, g, h, i, n_keys, s_buf);
+    const uint16_t *doi = dO + ((tok0 + i) * p->Hq + h) * (int64_t)D;
+    double delta = 0.0;
+    for (int j = 0; j < n_keys; ++j) {
+        const uint16_t *vj = p->v + ((tok0 + j) * p->Hkv + g) * (int64_t)D;
+        double dp = 0.0;
+        for (int d = 0; d < D; ++d)
+            dp += bf16_bits_to_f64(doi[d]) * bf16_bits_to_f64(vj[d]);
+        s_buf[j] = exp(s_buf[j] - lse);
+        dp_buf[j] = dp;
+        delta += s_buf[j] * dp;
+    }
+    return delta;
+}
+
+static int keys_of_row(const problem_t *p, int i, int L)
+{
+    return p->causal ? (i + 1 < L ? i + 1 : L) : L; /* |K_i| */
+}
+
+static void *bwd_worker(void *arg)
+{
+    bwd_job_t *job = (bwd_job_t *)arg;
+    const problem_t *p = job->p;
+    const int D = p->D, group = p->Hq / p->Hkv;
+    const size_t n = (size_t)(job->max_len > 0 ? job->max_len : 1);
+    double *s_buf = (double *)malloc(sizeof(double) * n);
+    double *dp_buf = (double *)malloc(sizeof(double) * n);
+    if (!s_buf || !dp_buf) {
+        free(s_buf);
+        free(dp_buf);
+        return NULL;
+    }
+    for (;;) {
+        int64_t t = __atomic_fetch_add(job->next, 1, __ATOMIC_RELAXED);
+        if (t >= job->n_tasks)
+            break;
+        const int b = (int)(t / p->Hkv), g = (int)(t % p->Hkv);
+        int64_t tok0;
+        int L;
+        seq_bounds(p, b, &tok0, &L);
+        for (int j = 0; j < L; ++j)
+            for (int d = 0; d < D; ++d) {
+                job->dk[((tok0 + j) * p->Hkv + g) * (int64_t)D + d] = 0.0;
+                job->dv[((tok0 + j) * p->Hkv + g) * (int64_t)D + d] = 0.0;
+            }
+        for (int h = g * group; h < (g + 1) * group; ++h) {
+            for (int i = 0; i < L; ++i) {
+                const int n_keys = keys_of_row(p, i, L);
+                double *dqi = job->dq + ((tok0 + i) * p->Hq + h) * (int64_t)D;
+                for (int d = 0; d < D; ++d)
+                    dqi[d] = 0.0;
+                if (n_keys == 0)
+                    continue;
+                const double delta = row_probs(p, job->dO, tok0, g, h, i, n_keys, s_buf, dp_buf);
+                const uint16_t *qi = p->q + ((tok0 + i) * p->Hq + h) * (int64_t)D;
+                const uint16_t *doi = job->dO + ((tok0 + i) * p->Hq + h) * (int64_t)D;
+                for (int j = 0; j < n_keys; ++j) {
+                    const double P = s_buf[j];
+                    const double dS = P * (dp_buf[j] - delta);
+                    const uint16_t *kj = p->k + ((tok0 + j) * p->Hkv + g) * (int64_t)D;
+                    double *dkj = job->dk + ((tok0 + j) * p->Hkv + g) * (int64_t)D;
+                    double *dvj = job->dv + ((tok0 + j) * p->Hkv + g) * (int64_t)D;
+                    for (int d = 0; d < D; ++d) {
+                        dqi[d] += p->scale * dS * bf16_bits_to_f64(kj[d]);
+                        dkj[d] += p->scale * dS * bf16_bits_to_f64(qi[d]);
+                        dvj[d] += P * bf16_bits_to_f64(doi[d]);
+                    }
+                }
+            }
+        }
+    }
+    free(s_buf);
+    free(dp_buf);
+    return NULL;
+}
+
+/*
+ * Full backward pass.  Tasks are (sequence, key/value head) pairs: one thread
+ * owns the dk, dv rows of its head and the dq rows of the head's query group,
+ * so no two threads write the same element.
+ */
+int mk_oracle_attn_bwd_f64(const uint16_t *q, const uint16_t *k, const uint16_t *v,
+                           const uint16_t *dO, double *dq, double *dk, double *dv, int B,
+                           int Hq, int Hkv, int S, int D, int causal, double scale,
+                           const int32_t *cu_seqlens, int n_threads)
+{
+    problem_t p = {q, k, v, B, Hq, Hkv, S, D, causal != 0, scale, cu_seqlens};
+    int st = check_problem(&p);
+    if (st != MK_ORACLE_OK)
+        return st;
+    if (!dO || !dq || !dk || !dv)
+        return MK_ORACLE_BAD_ARG;
+    int64_t next = 0;
+    bwd_job_t job = {&p, dO, dq, dk, dv, (int64_t)B * Hkv, &next, max_seq_len(&p)};
+    return run_threads(bwd_worker, &job, sizeof job, n_threads);
+}
+
+/* ---------------------------------------------------- sampled backward parts */
+
+typedef struct {
+    const problem_t *p;
+    const uint16_t *dO;
+    const int64_t *items; /* dq rows: (b, h, i); dk/dv ranges: (b, g, j0, j1) */
+    double *out0, *out1;  /* dq rows; or dk, dv rows of the ranges, in order */
+    const int64_t *out_off; /* ranges: first output row of each range */
+    int64_t n_items;
+    int64_t *next;
+    int max_len;
+} bwd_sample_job_t;
+
+static void *dq_rows_worker(void *arg)
+{
+    bwd_sample_job_t *job = (bwd_sample_job_t *)arg;
+    const problem_t *p = job->p;
+    const int D = p->D, group = p->Hq / p->Hkv;
+    const size_t n = (size_t)(job->max_len > 0 ? job->max_len : 1);
+    double *s_buf = (double *)malloc(sizeof(double) * n);
+    double *dp_buf = (double *)malloc(sizeof(double) * n);
+    if (!s_buf || !dp_buf) {
+        free(s_buf);
+        free(dp_buf);
+        return NULL;
+    }
+    for (;;) {
+        int64_t r = __atomic_fetch_add(job->next, 1, __ATOMIC_RELAXED);
+        if (r >= job->n_items)
+            break;
+        const int b = (int)job->items[3 * r], h = (int)job->items[3 * r + 1];
+        const int i = (int)job->items[3 * r + 2], g = h / group;
+        int64_t tok0;
+        int L;
+        seq_bounds(p, b, &tok0, &L);
+        const int n_keys = keys_of_row(p, i, L);
+        double *dqi = job->out0 + r * (int64_t)D;
+        for (int d = 0; d < D; ++d)
+            dqi[d] = 0.0;
+        if (n_keys == 0)
+            continue;
+        const double delta = row_probs(p, job->dO, tok0, g, h, i, n_keys, s_buf, dp_buf);
+        for (int j = 0; j < n_keys; ++j) {
+            const double dS = s_buf[j] * (dp_buf[j] - delta);
+            const uint16_t *kj = p->k + ((tok0 + j) * p->Hkv + g) * (int64_t)D;
+            for (int d = 0; d < D; ++d)
+                dqi[d] += p->scale * dS * bf16_bits_to_f64(kj[d]);
+        }
+    }
+    free(s_buf);
+    free(dp_buf);
+    return NULL;
+}
+
+/*
+ * dq on selected rows (b, h, i) only.  dq of a row depends on that row's
+ * scores alone, so a sampled row equals the row of mk_oracle_attn_bwd_f64.
+ */
+int mk_oracle_attn_bwd_dq_rows_f64(const uint16_t *q, const uint16_t *k, const uint16_t *v,
+                                   const uint16_t *dO, int B, int Hq, int Hkv, int S, int D,
+                                   int causal, double scale, const int32_t *cu_seqlens,
+                                   const int64_t *rows, int64_t n_rows, double *dq_rows,
+                                   int n_threads)
+{
+    problem_t p = {q, k, v, B, Hq, Hkv, S, D, causal != 0, scale, cu_seqlens};
+    int st = check_problem(&p);
+    if (st != MK_ORACLE_OK)
+        return st;
+    if (!dO || n_rows < 0 || (n_rows > 0 && (!rows || !dq_rows)))
+        return MK_ORACLE_BAD_ARG;
+    for (int64_t r = 0; r < n_rows; ++r) {
+        int b = (int)rows[3 * r], h = (int)rows[3 * r + 1], i = (int)rows[3 * r + 2];
+        if (b < 0 || b >= B || h < 0 || h >= Hq || i < 0)
+            return MK_ORACLE_BAD_ARG;
+        int64_t t0;
+        int L;
+        seq_bounds(&p, b, &t0, &L);
+        if (i >= L)
+            return MK_ORACLE_BAD_ARG;
+    }
+    int64_t next = 0;
+    bwd_sample_job_t job = {&p, dO, rows, dq_rows, NULL, NULL, n_rows, &next, max_seq_len(&p)};
+    return run_threads(dq_rows_worker, &job, sizeof job, n_threads);
+}
+
+static void *dkv_range_worker(void *arg)
+{
+    bwd_sample_job_t *job = (bwd_sample_job_t *)arg;
+    const problem_t *p = job->p;
+    const int D = p->D, group = p->Hq / p->Hkv;
+    const size_t n = (size_t)(job->max_len > 0 ? job->max_len : 1);
+    double *s_buf = (double *)malloc(sizeof(double) * n);
+    double *dp_buf = (double *)malloc(sizeof(double) * n);
+    if (!s_buf || !dp_buf) {
+        free(s_buf);
+        free(dp_buf);
+        return NULL;
+    }
+    for (;;) {
+        int64_t r = __atomic_fetch_add(job->next, 1, __ATOMIC_RELAXED);
+        if (r >= job->n_items)
+            break;
+        const int b = (int)job->items[4 * r], g = (int)job->items[4 * r + 1];
+        const int j0 = (int)job->items[4 * r + 2], j1 = (int)job->items[4 * r + 3];
+        int64_t tok0;
+        int L;
+        seq_bounds(p, b, &tok0, &L);
+        double *dk = job->out0 + job->out_off[r] * (int64_t)D;
+        double *dv = job->out1 + job->out_off[r] * (int64_t)D;
+        for (int64_t e = 0; e < (int64_t)(j1 - j0) * D; ++e)
+            dk[e] = dv[e] = 0.0;
+        /* Every query row that sees a key of [j0, j1): all rows, or rows
+         * i >= j0 when causal. */
+        for (int h = g * group; h < (g + 1) * group; ++h) {
+            for (int i = p->causal ? j0 : 0; i < L; ++i) {
+                const int n_keys = keys_of_row(p, i, L);
+                if (n_keys <= j0)
+                    continue;
+                const double delta = row_probs(p, job->dO, tok0, g, h, i, n_keys, s_buf, dp_buf);
+                const uint16_t *qi = p->q + ((tok0 + i) * p->Hq + h) * (int64_t)D;
+                const uint16_t *doi = job->dO + ((tok0 + i) * p->Hq + h) * (int64_t)D;
+                for (int j = j0; j < j1 && j < n_keys; ++j) {
+                    const double P = s_buf[j];
+                    const double dS = P * (dp_buf[j] - delta);
+                    for (int d = 0; d < D; ++d) {
+                        dk[(int64_t)(j - j0) * D + d] += p->scale * dS * bf16_bits_to_f64(qi[d]);
+                        dv[(int64_t)(j - j0) * D + d] += P * bf16_bits_to_f64(doi[d]);
+                    }
+                }
+            }
+        }
+    }
+    free(s_buf);
+    free(dp_buf);
+    return NULL;
+}
+
+/*
+ * dk and dv for key ranges [j0, j1) of (sequence b, key/value head g), given
+ * as n_ranges x 4 int64 (b, g, j0, j1); the ranges' rows are written one
+ * after the other into dk_rows and dv_rows (sum of (j1 - j0) rows of D).
+ * Each range visits every query row that sees one of its keys, so it equals
+ * the same rows of mk_oracle_attn_bwd_f64.
+ */
+int mk_oracle_attn_bwd_dkv_ranges_f64(const uint16_t *q, const uint16_t *k, const uint16_t *v,
+                                      const uint16_t *dO, int B, int Hq, int Hkv, int S, int D,
+                                      int causal, double scale, const int32_t *cu_seqlens,
+                                      const int64_t *ranges, int64_t n_ranges, double *dk_rows,
+                                      double *dv_rows, int n_threads)
+{
+    problem_t p = {q, k, v, B, Hq, Hkv, S, D, causal != 0, scale, cu_seqlens};
+    int st = check_problem(&p);
+    if (st != MK_ORACLE_OK)
+        return st;
+    if (!dO || n_ranges < 0 || (n_ranges > 0 && (!ranges || !dk_rows || !dv_rows)))
+        return MK_ORACLE_BAD_ARG;
+    int64_t *off = (int64_t *)malloc(sizeof(int64_t) * (size_t)(n_ranges > 0 ? n_ranges : 1));
+    if (!off)
+        return MK_ORACLE_NO_MEM;
+    int64_t rows = 0;
+    for (int64_t r = 0; r < n_ranges; ++r) {
+        const int64_t b = ranges[4 * r], g = ranges[4 * r + 1];
+        const int64_t j0 = ranges[4 * r + 2], j1 = ranges[4 * r + 3];
+        int64_t t0;
+        int L = 0;
+        if (b >= 0 && b < B)
+            seq_bounds(&p, (int)b, &t0, &L);
+        if (b < 0 || b >= B || g < 0 || g >= Hkv || j0 < 0 || j1 < j0 || j1 > L) {
+            free(off);
+            return MK_ORACLE_BAD_ARG;
+        }
+        off[r] = rows;
+        rows += j1 - j0;
+    }
+    int64_t next = 0;
+    bwd_sample_job_t job = {&p, dO, ranges, dk_rows, dv_rows, off, n_ranges, &next, max_seq_len(&p)};
+    st = run_threads(dkv_range_worker, &job, sizeof job, n_threads);
+    free(off);
+    return st;
 }

@@ -126,6 +126,14 @@ def make_qkv(B: int, Hq: int, Hkv: int, S: int, D: int, seed: int, sigma: float 
     return q, k, v, cu
 
 
+def make_grad_out(shape, seed: int, sigma: float = 1.0) -> torch.Tensor:
+    """Seeded bf16 output gradient dO for the backward pass (layout of q):
+    N(0, sigma^2) drawn from its own generator, so that q, k, v of the same
+    seed are unchanged."""
+    g = torch.Generator("cpu").manual_seed(seed + 7919)
+    return randn_bf16(tuple(shape), g, sigma)
+
+
 def plant_adversarial_rows(q32: torch.Tensor, k32: torch.Tensor, scale: float, seed: int,
                            n_rows: int = 4, gap: float = 30.0, noise: float = 1e-3):
     """Makes, in each (b, h), `n_rows` query rows whose logit row has one entry

@@ -399,6 +399,216 @@ def check_decode_empty_sequence(lib):
     assert np.all(np.isfinite(lse[1])), "non-empty sequence lse"
 
 
+# --------------------------------------------------------------- backward pass
+
+def _bwd(lib, q, k, v, do, causal, scale, cu=None):
+    return oracle.attn_bwd(q, k, v, do, causal, scale, cu_seqlens=cu, n_threads=2, lib=lib)
+
+
+def _fwd_loss_f64(q, k, v, do, causal, scale, seqs):
+    """sum(o * do) for fp64 q [T,Hq,D], k/v [T,Hkv,D], do [T,Hq,D], through
+    the brute-force explicit-P forward (no gradient formula involved)."""
+    Hq, Hkv = q.shape[1], k.shape[1]
+    G = Hq // Hkv
+    loss = 0.0
+    for t0, L in seqs:
+        for h in range(Hq):
+            g = h // G
+            P = brute.probability_matrix(q[t0:t0 + L, h], k[t0:t0 + L, g], causal, scale)
+            loss += float(np.sum((P @ v[t0:t0 + L, g]) * do[t0:t0 + L, h]))
+    return loss
+
+
+def check_bwd_finite_differences(lib):
+    """Directional derivatives of sum(o * dO) by central differences of the
+    brute-force forward (fp64, step 1e-5) equal <grad, direction> from the
+    oracle's dq, dk, dv: fixed length and varlen, causal or not, GQA."""
+    rng = np.random.default_rng(5)
+    cases = [
+        dict(B=1, Hq=4, Hkv=2, S=6, D=4, causal=True, lens=None),
+        dict(B=2, Hq=3, Hkv=1, S=5, D=3, causal=False, lens=None),
+        dict(B=0, Hq=2, Hkv=2, S=0, D=4, causal=True, lens=[3, 1, 4]),
+    ]
+    for n, c in enumerate(cases):
+        q, k, v, cu = W.make_qkv(c["B"], c["Hq"], c["Hkv"], c["S"], c["D"], seed=61 + n,
+                                 lengths=c["lens"])
+        do = W.make_grad_out(q.shape, seed=61 + n)
+        scale = 0.45
+        cu_np = None if cu is None else cu.numpy()
+        dq, dk, dv = _bwd(lib, q, k, v, do, c["causal"], scale, cu_np)
+        if cu is None:
+            B, S = c["B"], c["S"]
+            seqs = [(b * S, S) for b in range(B)]
+            flat = lambda t: _f64(t).reshape(B * S, t.shape[2], t.shape[3])
+        else:
+            seqs = [(int(cu[b]), int(cu[b + 1] - cu[b])) for b in range(len(cu) - 1)]
+            flat = _f64
+        x = [flat(q), flat(k), flat(v)]
+        g = [dq.reshape(x[0].shape), dk.reshape(x[1].shape), dv.reshape(x[2].shape)]
+        dof = flat(do)
+        eps = 1e-5
+        for t in range(4):
+            dirs = [rng.standard_normal(a.shape) for a in x]
+            plus = [a + eps * d for a, d in zip(x, dirs)]
+            minus = [a - eps * d for a, d in zip(x, dirs)]
+            fd = (_fwd_loss_f64(*plus, dof, c["causal"], scale, seqs) -
+                  _fwd_loss_f64(*minus, dof, c["causal"], scale, seqs)) / (2 * eps)
+            an = sum(float(np.sum(gg * d)) for gg, d in zip(g, dirs))
+            assert abs(fd - an) <= 1e-7 * max(1.0, abs(an)), \
+                f"bwd finite differences case {n}: {fd!r} vs {an!r}"
+            # one operand at a time, so that a mistake in one gradient cannot
+            # hide behind another
+            for w in range(3):
+                pl = list(x)
+                mi = list(x)
+                pl[w] = x[w] + eps * dirs[w]
+                mi[w] = x[w] - eps * dirs[w]
+                fd_w = (_fwd_loss_f64(*pl, dof, c["causal"], scale, seqs) -
+                        _fwd_loss_f64(*mi, dof, c["causal"], scale, seqs)) / (2 * eps)
+                an_w = float(np.sum(g[w] * dirs[w]))
+                assert abs(fd_w - an_w) <= 1e-7 * max(1.0, abs(an_w)), \
+                    f"bwd finite differences case {n} operand {w}: {fd_w!r} vs {an_w!r}"
+
+
+def check_bwd_torch_autograd(lib):
+    """Library special case: reverse-mode autograd of PyTorch's fp64
+    scaled_dot_product_attention on CPU (K/V repeated per group for GQA, so
+    autograd sums each group's gradients)."""
+    for causal in (True, False):
+        B, Hq, Hkv, S, D = 2, 6, 2, 11, 8
+        q, k, v, _ = W.make_qkv(B, Hq, Hkv, S, D, seed=71 + int(causal))
+        do = W.make_grad_out(q.shape, seed=71 + int(causal))
+        scale = 0.3
+        dq, dk, dv = _bwd(lib, q, k, v, do, causal, scale)
+        G = Hq // Hkv
+        qt = torch.from_numpy(_f64(q)).permute(0, 2, 1, 3).requires_grad_()
+        kt = torch.from_numpy(_f64(k)).permute(0, 2, 1, 3).requires_grad_()
+        vt = torch.from_numpy(_f64(v)).permute(0, 2, 1, 3).requires_grad_()
+        o = torch.nn.functional.scaled_dot_product_attention(
+            qt, kt.repeat_interleave(G, dim=1), vt.repeat_interleave(G, dim=1),
+            is_causal=causal, scale=scale)
+        o.backward(torch.from_numpy(_f64(do)).permute(0, 2, 1, 3))
+        _close(dq, qt.grad.permute(0, 2, 1, 3).numpy(), 1e-12, f"autograd dq causal={causal}")
+        _close(dk, kt.grad.permute(0, 2, 1, 3).numpy(), 1e-12, f"autograd dk causal={causal}")
+        _close(dv, vt.grad.permute(0, 2, 1, 3).numpy(), 1e-12, f"autograd dv causal={causal}")
+
+
+def check_bwd_zero_scale(lib):
+    """scale = 0: P is uniform over the visible keys and no logit depends on
+    q or k, so dq = dk = 0 exactly and dv_j = sum over the group's heads and
+    the rows i that see j of dO_i / |K_i|."""
+    B, Hq, Hkv, S, D = 2, 4, 2, 9, 4
+    q, k, v, _ = W.make_qkv(B, Hq, Hkv, S, D, seed=81)
+    do = W.make_grad_out(q.shape, seed=81)
+    G = Hq // Hkv
+    dof = _f64(do)
+    for causal in (True, False):
+        dq, dk, dv = _bwd(lib, q, k, v, do, causal, 0.0)
+        assert np.all(dq == 0.0) and np.all(dk == 0.0), "scale 0: dq, dk not zero"
+        want = np.zeros_like(dv)
+        for b in range(B):
+            for g in range(Hkv):
+                for j in range(S):
+                    rows = range(j, S) if causal else range(S)
+                    for h in range(g * G, (g + 1) * G):
+                        for i in rows:
+                            want[b, j, g] += dof[b, i, h] / ((i + 1) if causal else S)
+        _close(dv, want, 1e-13, f"scale 0 dv causal={causal}")
+
+
+def check_bwd_single_key(lib):
+    """S = 1: P = 1 whatever the logit, so dq = dk = 0 and dv_0 is the sum of
+    dO_0 over the group's heads."""
+    B, Hq, Hkv, D = 2, 6, 3, 8
+    q, k, v, _ = W.make_qkv(B, Hq, Hkv, 1, D, seed=91)
+    do = W.make_grad_out(q.shape, seed=91)
+    for causal in (True, False):
+        dq, dk, dv = _bwd(lib, q, k, v, do, causal, 0.8)
+        _close(dq, np.zeros_like(dq), 1e-15, "single key dq")
+        _close(dk, np.zeros_like(dk), 1e-15, "single key dk")
+        want = _f64(do).reshape(B, 1, Hkv, Hq // Hkv, D).sum(axis=3)
+        _close(dv, want, 1e-14, "single key dv")
+
+
+def check_bwd_sum_identities(lib):
+    """Every row of dS sums to zero (sum_j P_ij (dP_ij - Delta_i) = Delta_i -
+    Delta_i), so sum_j dk_j = 0 for each (sequence, key/value head); and the
+    rows of P sum to one, so sum_j dv_j = sum over the group's heads and all
+    rows of dO_i."""
+    lens = [7, 1, 12]
+    q, k, v, cu = W.make_qkv(0, 6, 2, 0, 8, seed=101, lengths=lens)
+    do = W.make_grad_out(q.shape, seed=101)
+    G = 3
+    for causal in (True, False):
+        dq, dk, dv = _bwd(lib, q, k, v, do, causal, 0.6, cu.numpy())
+        dof = _f64(do)
+        for b in range(len(lens)):
+            t0, t1 = int(cu[b]), int(cu[b + 1])
+            for g in range(2):
+                _close(dk[t0:t1, g].sum(axis=0), np.zeros(8), 1e-12, "sum of dk")
+                want = dof[t0:t1, g * G:(g + 1) * G].sum(axis=(0, 1))
+                _close(dv[t0:t1, g].sum(axis=0), want, 1e-12, "sum of dv")
+        assert np.max(np.abs(dk)) > 1e-3, "dk identically zero"
+
+
+def check_bwd_gqa_equals_repeated_mha(lib):
+    """GQA equals MHA on K/V repeated per group, with dk, dv summed over the
+    group's copies."""
+    B, Hq, Hkv, S, D = 2, 8, 2, 10, 4
+    q, k, v, _ = W.make_qkv(B, Hq, Hkv, S, D, seed=111)
+    do = W.make_grad_out(q.shape, seed=111)
+    G = Hq // Hkv
+    kr = k.repeat_interleave(G, dim=2).contiguous()
+    vr = v.repeat_interleave(G, dim=2).contiguous()
+    for causal in (True, False):
+        dq, dk, dv = _bwd(lib, q, k, v, do, causal, 0.5)
+        dq2, dk2, dv2 = _bwd(lib, q, kr, vr, do, causal, 0.5)
+        _close(dq, dq2, 1e-13, "gqa dq")
+        _close(dk, dk2.reshape(B, S, Hkv, G, D).sum(axis=3), 1e-13, "gqa dk")
+        _close(dv, dv2.reshape(B, S, Hkv, G, D).sum(axis=3), 1e-13, "gqa dv")
+
+
+def check_bwd_varlen_equals_separate(lib):
+    """A packed varlen batch equals one fixed-length call per sequence."""
+    lens = [5, 9, 1, 4]
+    q, k, v, cu = W.make_qkv(0, 4, 2, 0, 8, seed=121, lengths=lens)
+    do = W.make_grad_out(q.shape, seed=121)
+    for causal in (True, False):
+        dq, dk, dv = _bwd(lib, q, k, v, do, causal, 0.4, cu.numpy())
+        for b, L in enumerate(lens):
+            t0 = int(cu[b])
+            sl = slice(t0, t0 + L)
+            e = _bwd(lib, q[sl][None].contiguous(), k[sl][None].contiguous(),
+                     v[sl][None].contiguous(), do[sl][None].contiguous(), causal, 0.4)
+            _close(dq[sl], e[0][0], 1e-13, "varlen dq")
+            _close(dk[sl], e[1][0], 1e-13, "varlen dk")
+            _close(dv[sl], e[2][0], 1e-13, "varlen dv")
+
+
+def check_bwd_sampled_match_full(lib):
+    """The sampled forms (dq on rows, dk / dv on key ranges) equal the same
+    rows of the full backward pass."""
+    for causal in (True, False):
+        lens = [13, 6, 20]
+        q, k, v, cu = W.make_qkv(0, 6, 3, 0, 8, seed=131, lengths=lens)
+        do = W.make_grad_out(q.shape, seed=131)
+        dq, dk, dv = _bwd(lib, q, k, v, do, causal, 0.35, cu.numpy())
+        rows = [(0, 0, 0), (0, 5, 12), (1, 2, 3), (2, 4, 19), (2, 1, 7)]
+        got = oracle.attn_bwd_dq_rows(q, k, v, do, causal, 0.35, rows, cu_seqlens=cu.numpy(),
+                                      n_threads=2, lib=lib)
+        for r, (b, h, i) in enumerate(rows):
+            _close(got[r], dq[int(cu[b]) + i, h], 1e-13, "sampled dq row")
+        ranges = [(0, 1, 0, 13), (2, 0, 17, 20), (1, 2, 2, 3), (2, 2, 5, 11)]
+        gk, gv = oracle.attn_bwd_dkv_ranges(q, k, v, do, causal, 0.35, ranges,
+                                            cu_seqlens=cu.numpy(), n_threads=2, lib=lib)
+        at = 0
+        for b, g, j0, j1 in ranges:
+            t0 = int(cu[b])
+            _close(gk[at:at + j1 - j0], dk[t0 + j0:t0 + j1, g], 1e-13, "sampled dk range")
+            _close(gv[at:at + j1 - j0], dv[t0 + j0:t0 + j1, g], 1e-13, "sampled dv range")
+            at += j1 - j0
+
+
 ALL_CHECKS = [
     check_brute_force_tiny,
     check_brute_force_varlen,
@@ -421,4 +631,12 @@ ALL_CHECKS = [
     check_decode_single_key,
     check_decode_identical_keys,
     check_decode_empty_sequence,
+    check_bwd_finite_differences,
+    check_bwd_torch_autograd,
+    check_bwd_zero_scale,
+    check_bwd_single_key,
+    check_bwd_sum_identities,
+    check_bwd_gqa_equals_repeated_mha,
+    check_bwd_varlen_equals_separate,
+    check_bwd_sampled_match_full,
 ]

@@ -40,6 +40,28 @@ MUTANTS = {
     "decode_interleaved_groups": ("h = (int)(t % job->Hq), g = h / G;", "h = (int)(t % job->Hq), g = h % job->Hkv;"),
     "decode_drop_scale": ("s_buf[j] = job->scale * acc;", "s_buf[j] = acc;"),
     "decode_lse_log2": ("job->lse[t] = m + log(l);", "job->lse[t] = m + log2(l);"),
+    "bwd_drop_delta": ("const double dS = P * (dp_buf[j] - delta);\n                    const uint16_t *kj",
+                       "const double dS = P * dp_buf[j];\n                    const uint16_t *kj"),
+    "bwd_delta_sign": ("delta += s_buf[j] * dp;", "delta -= s_buf[j] * dp;"),
+    "bwd_dk_without_scale": ("dkj[d] += p->scale * dS * bf16_bits_to_f64(qi[d]);",
+                             "dkj[d] += dS * bf16_bits_to_f64(qi[d]);"),
+    "bwd_dk_from_keys": ("dkj[d] += p->scale * dS * bf16_bits_to_f64(qi[d]);",
+                         "dkj[d] += p->scale * dS * bf16_bits_to_f64(kj[d]);"),
+    "bwd_dq_from_queries": ("dqi[d] += p->scale * dS * bf16_bits_to_f64(kj[d]);\n                        dkj",
+                            "dqi[d] += p->scale * dS * bf16_bits_to_f64(qi[d]);\n                        dkj"),
+    "bwd_dv_uses_ds": ("dvj[d] += P * bf16_bits_to_f64(doi[d]);", "dvj[d] += dS * bf16_bits_to_f64(doi[d]);"),
+    "bwd_dv_uses_queries": ("dvj[d] += P * bf16_bits_to_f64(doi[d]);", "dvj[d] += P * bf16_bits_to_f64(qi[d]);"),
+    "bwd_dp_from_keys": ("const uint16_t *vj = p->v + ((tok0 + j) * p->Hkv + g) * (int64_t)D;\n        double dp",
+                         "const uint16_t *vj = p->k + ((tok0 + j) * p->Hkv + g) * (int64_t)D;\n        double dp"),
+    "bwd_probs_without_lse": ("s_buf[j] = exp(s_buf[j] - lse);", "s_buf[j] = exp(s_buf[j]);"),
+    "bwd_first_head_only": ("for (int h = g * group; h < (g + 1) * group; ++h) {\n            for (int i = 0; i < L; ++i) {",
+                            "for (int h = g * group; h < g * group + 1; ++h) {\n            for (int i = 0; i < L; ++i) {"),
+    "bwd_causal_excludes_diagonal": ("return p->causal ? (i + 1 < L ? i + 1 : L) : L; /* |K_i| */",
+                                     "return p->causal ? (i < L ? i : L) : L; /* |K_i| */"),
+    "bwd_dq_rows_drop_scale": ("dqi[d] += p->scale * dS * bf16_bits_to_f64(kj[d]);\n        }\n    }",
+                               "dqi[d] += dS * bf16_bits_to_f64(kj[d]);\n        }\n    }"),
+    "bwd_ranges_skip_first_row": ("for (int i = p->causal ? j0 : 0; i < L; ++i) {",
+                                  "for (int i = p->causal ? j0 + 1 : 0; i < L; ++i) {"),
 }
 
 
