@@ -25,15 +25,17 @@ MUTANTS = {
     "causal_ignored": ("int n_keys = p->causal ? (i + 1 < L ? i + 1 : L) : L;",
                        "int n_keys = L;"),
     "gqa_interleaved_groups": ("const int g = h / group;", "const int g = h % p->Hkv;"),
-    "keys_read_from_values": ("const uint16_t *kj = p->k + ", "const uint16_t *kj = p->v + "),
-    "values_read_from_keys": ("const uint16_t *vj = p->v + ", "const uint16_t *vj = p->k + "),
-    "query_row_offset": ("const uint16_t *qi = p->q + ((tok0 + i) * p->Hq + h)",
-                         "const uint16_t *qi = p->q + ((tok0 + i) * p->Hq + 0)"),
+    "keys_read_from_values": ("/* |K_i| */\n\n    double m = -INFINITY;\n    for (int j = 0; j < n_keys; ++j) {\n        const uint16_t *kj = p->k + ",
+                              "/* |K_i| */\n\n    double m = -INFINITY;\n    for (int j = 0; j < n_keys; ++j) {\n        const uint16_t *kj = p->v + "),
+    "values_read_from_keys": ("const uint16_t *vj = p->v + ((tok0 + j) * p->Hkv + g) * (int64_t)D;\n        double w",
+                              "const uint16_t *vj = p->k + ((tok0 + j) * p->Hkv + g) * (int64_t)D;\n        double w"),
+    "query_row_offset": ("const uint16_t *qi = p->q + ((tok0 + i) * p->Hq + h) * (int64_t)D;\n    int n_keys",
+                         "const uint16_t *qi = p->q + ((tok0 + i) * p->Hq + 0) * (int64_t)D;\n    int n_keys"),
     "varlen_lse_index": ("int64_t lse_idx = p->cu ? (int64_t)h * p->S + tok0 + i",
                          "int64_t lse_idx = p->cu ? (int64_t)h * p->S + i"),
     "weights_not_accumulated": ("        l += w;\n", "        l = w;\n"),
-    "last_dim_dropped": ("for (int d = 0; d < D; ++d)\n            dot +=",
-                         "for (int d = 0; d + 1 < D; ++d)\n            dot +="),
+    "last_dim_dropped": ("for (int d = 0; d < D; ++d)\n            dot += bf16_bits_to_f64(qi[d]) * bf16_bits_to_f64(kj[d]);\n        double s",
+                         "for (int d = 0; d + 1 < D; ++d)\n            dot += bf16_bits_to_f64(qi[d]) * bf16_bits_to_f64(kj[d]);\n        double s"),
     "decode_slot_from_page_index": (
         "const int64_t row = (page * job->page_size + j % job->page_size) * job->Hkv + g;\n            const uint16_t *kr",
         "const int64_t row = (page * job->page_size + j / job->page_size) * job->Hkv + g;\n            const uint16_t *kr"),
