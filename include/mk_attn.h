@@ -1,5 +1,6 @@
 /*
- * mk_attn.h -- C ABI of the GB300 (sm_103a) attention forward library.
+ * mk_attn.h -- C ABI of the GB300 (sm_103a) attention library: forward and
+ * backward passes and a paged decode step.
  *
  * The operation is the fused attention forward pass whose reference the
  * paper's Flash Attention and GQA Attention kernels reproduce (Table 2; the
@@ -101,6 +102,50 @@ MK_API int mk_attn_fwd_stall_test(const void *q, const void *k, const void *v, v
                                   float scale, const int32_t *cu_seqlens, void *stream);
 
 /*
+ * mk_attn_bwd_workspace_bytes -- bytes of device workspace mk_attn_bwd needs
+ * (one fp32 per query row and head: Delta_i = dO_i . o_i), or -1 for invalid
+ * sizes.  varlen: nonzero when cu_seqlens will be passed (S = total tokens).
+ */
+MK_API int64_t mk_attn_bwd_workspace_bytes(int B, int Hq, int S, int varlen);
+
+/*
+ * mk_attn_bwd -- attention backward pass: the gradients of the mk_attn_fwd
+ * operation with respect to q, k and v for an output gradient dO (the
+ * training step of the paper's attention kernels, Table 2).  With
+ * P_ij = exp(scale * q_i . k_j - lse_i) over the keys row i sees:
+ *   dv_j = sum_{h in group(j)} sum_i P_ij dO_i
+ *   dS_ij = P_ij (dO_i . v_j - Delta_i),   Delta_i = dO_i . o_i
+ *   dq_i = scale * sum_j dS_ij k_j
+ *   dk_j = scale * sum_{h in group(j)} sum_i dS_ij q_i
+ *
+ * Arguments (all pointers are DEVICE pointers owned by the caller):
+ *   q, k, v, B, Hq, Hkv, S, D, causal, scale, cu_seqlens
+ *              exactly as passed to mk_attn_fwd.
+ *   o, lse     the outputs of that mk_attn_fwd call (bf16 o, fp32 lse).
+ *   dO         bf16 gradient of o, layout of q.  Read only.
+ *   dq         bf16 output, layout of q.  Fully overwritten.
+ *   dk, dv     bf16 outputs, layout of k and v.  Fully overwritten; rows of
+ *              keys that no query sees are zero.
+ *   workspace  device buffer of at least mk_attn_bwd_workspace_bytes()
+ *              bytes, 16-byte aligned; scratch, contents on entry do not
+ *              matter.  Calls that share a workspace must not overlap.
+ *   stream     cudaStream_t; three kernels are enqueued (Delta, dK/dV, dQ),
+ *              the call never synchronises.
+ * Layout and alignment: as mk_attn_fwd; dO, dq, dk, dv and workspace 16-byte
+ * aligned, lse 4-byte aligned.
+ * Returns MK_OK, or MK_ERR_INVALID_ARG (null pointer, sizes, too small a
+ * workspace), MK_ERR_UNSUPPORTED (D), MK_ERR_ALIGNMENT, MK_ERR_CUDA; on any
+ * error nothing is enqueued.  Deterministic: no atomics, repeated calls give
+ * bitwise identical gradients.  Internal waits are bounded as in mk_attn_fwd
+ * (MK_ERR_TIMEOUT through mk_attn_check_status).
+ */
+MK_API int mk_attn_bwd(const void *q, const void *k, const void *v, const void *o,
+                       const float *lse, const void *dO, void *dq, void *dk, void *dv, int B,
+                       int Hq, int Hkv, int S, int D, int causal, float scale,
+                       const int32_t *cu_seqlens, void *workspace, int64_t workspace_bytes,
+                       void *stream);
+
+/*
  * mk_attn_decode_workspace_bytes -- bytes of device workspace that
  * mk_attn_decode_paged needs for these sizes on the current device (0: none),
  * or -1 for invalid sizes.  Depends on the device's SM count only through the
@@ -194,8 +239,9 @@ MK_API const char *mk_attn_error_string(int status);
 
 /*
  * mk_attn_check_status -- synchronises `stream`, then reads and clears the
- * device status words written by kernels whose internal waits ran out or
- * that met device-side inputs out of range (decode page tables, lengths).
+ * device status words written by kernels (forward, backward, decode) whose
+ * internal waits ran out or that met device-side inputs out of range (decode
+ * page tables, lengths).
  * Returns MK_OK, MK_ERR_TIMEOUT, MK_ERR_INVALID_ARG, or MK_ERR_CUDA if
  * synchronisation failed.
  */

@@ -25,7 +25,8 @@ MK_ERR_SCRATCH_LIMIT = -6
 DECODE_STATIC_SCRATCH_BYTES = 8 * 1024 * 1024
 
 # Symbols declared in include/mk_attn.h.
-EXPORTED = ("mk_attn_fwd", "mk_attn_fwd_stall_test", "mk_attn_decode_workspace_bytes",
+EXPORTED = ("mk_attn_fwd", "mk_attn_fwd_stall_test", "mk_attn_bwd_workspace_bytes", "mk_attn_bwd",
+            "mk_attn_decode_workspace_bytes",
             "mk_attn_decode_paged", "mk_attn_decode_paged_noalloc", "mk_attn_error_string",
             "mk_attn_check_status", "mk_attn_version")
 
@@ -60,6 +61,11 @@ def load_library() -> ctypes.CDLL:
             lib.mk_attn_fwd_stall_test.argtypes = lib.mk_attn_fwd.argtypes
             lib.mk_attn_fwd_stall_test.restype = i
             i64 = ctypes.c_int64
+            lib.mk_attn_bwd_workspace_bytes.argtypes = [i, i, i, i]
+            lib.mk_attn_bwd_workspace_bytes.restype = i64
+            lib.mk_attn_bwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, i, i, i, i, i, i,
+                                        ctypes.c_float, vp, vp, i64, vp]
+            lib.mk_attn_bwd.restype = i
             lib.mk_attn_decode_workspace_bytes.argtypes = [i, i, i, i, i, i]
             lib.mk_attn_decode_workspace_bytes.restype = i64
             lib.mk_attn_decode_paged.argtypes = [vp, vp, vp, vp, vp, vp, vp, i, i, i, i, i, i, i,
@@ -158,6 +164,74 @@ def attn_fwd(q, k, v, causal: bool = True, scale: float | None = None, cu_seqlen
                        B, Hq, Hkv, S, D, int(bool(causal)), float(scale), cu_ptr,
                        stream.cuda_stream))
     return out, lse
+
+
+def mk_attn_bwd_workspace_bytes(B: int, Hq: int, S: int, varlen: int) -> int:
+    return load_library().mk_attn_bwd_workspace_bytes(B, Hq, S, int(bool(varlen)))
+
+
+def mk_attn_bwd(q: int, k: int, v: int, o: int, lse: int, do: int, dq: int, dk: int, dv: int,
+                B: int, Hq: int, Hkv: int, S: int, D: int, causal: int, scale: float,
+                cu_seqlens: int | None, workspace: int | None, workspace_bytes: int,
+                stream: int | None) -> int:
+    """Raw C-ABI call: integer device pointers in, status code out."""
+    return load_library().mk_attn_bwd(q, k, v, o, lse, do, dq, dk, dv, B, Hq, Hkv, S, D,
+                                      int(causal), float(scale), cu_seqlens, workspace,
+                                      int(workspace_bytes), stream)
+
+
+def attn_bwd(q, k, v, o, lse, do, causal: bool = True, scale: float | None = None,
+             cu_seqlens=None, dq=None, dk=None, dv=None, workspace=None, stream=None):
+    """Attention backward on CUDA tensors through mk_attn_bwd.
+
+    q, k, v, causal, scale, cu_seqlens as for attn_fwd; o, lse its outputs;
+    do: bf16 gradient of o (layout of q).  Returns (dq, dk, dv), bf16, the
+    layouts of q, k, v.  PyTorch only allocates the outputs and the fp32
+    workspace and provides the stream."""
+    import torch
+    for name, t in (("q", q), ("k", k), ("v", v), ("o", o), ("do", do)):
+        if not t.is_cuda or t.dtype != torch.bfloat16 or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous bf16 CUDA tensor")
+    if not lse.is_cuda or lse.dtype != torch.float32 or not lse.is_contiguous():
+        raise ValueError("lse must be a contiguous fp32 CUDA tensor")
+    if o.shape != q.shape or do.shape != q.shape or k.shape != v.shape:
+        raise ValueError("o and do must have the shape of q, v that of k")
+    if cu_seqlens is None:
+        if q.dim() != 4:
+            raise ValueError("fixed-length layout is q [B,S,Hq,D], k/v [B,S,Hkv,D]")
+        B, S, Hq, D = q.shape
+        Hkv = k.shape[2]
+        lse_shape = (B, Hq, S)
+        cu_ptr = None
+    else:
+        if q.dim() != 3:
+            raise ValueError("varlen layout is q [T,Hq,D], k/v [T,Hkv,D]")
+        if not cu_seqlens.is_cuda or cu_seqlens.dtype != torch.int32 or cu_seqlens.dim() != 1:
+            raise ValueError("cu_seqlens must be a 1-D int32 CUDA tensor")
+        S, Hq, D = q.shape
+        Hkv = k.shape[1]
+        B = cu_seqlens.numel() - 1
+        lse_shape = (Hq, S)
+        cu_ptr = cu_seqlens.data_ptr()
+    if tuple(lse.shape) != lse_shape:
+        raise ValueError(f"lse must have shape {lse_shape}")
+    if scale is None:
+        scale = 1.0 / float(D) ** 0.5
+    dq = torch.empty_like(q) if dq is None else dq
+    dk = torch.empty_like(k) if dk is None else dk
+    dv = torch.empty_like(v) if dv is None else dv
+    need = mk_attn_bwd_workspace_bytes(B, Hq, S, cu_seqlens is not None)
+    if need < 0:
+        raise MkAttnError(MK_ERR_INVALID_ARG, "invalid backward sizes")
+    if workspace is None:
+        workspace = torch.empty((need + 15) // 16 * 4, dtype=torch.float32, device=q.device)
+    if stream is None:
+        stream = torch.cuda.current_stream(q.device)
+    _check(mk_attn_bwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), o.data_ptr(), lse.data_ptr(),
+                       do.data_ptr(), dq.data_ptr(), dk.data_ptr(), dv.data_ptr(), B, Hq, Hkv, S,
+                       D, int(bool(causal)), float(scale), cu_ptr, workspace.data_ptr(),
+                       workspace.numel() * workspace.element_size(), stream.cuda_stream))
+    return dq, dk, dv
 
 
 def mk_attn_decode_workspace_bytes(B: int, Hq: int, Hkv: int, D: int, page_size: int,

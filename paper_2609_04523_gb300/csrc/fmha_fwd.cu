@@ -869,6 +869,16 @@ static int launch(const void *q, const void *k, const void *v, const Params &p, 
 }  // namespace mk
 
 namespace mk {
+int fwd_take_status() {
+  int h = 0;
+  if (cudaMemcpyFromSymbol(&h, g_status, sizeof(int)) != cudaSuccess) return MK_ERR_CUDA;
+  if (h != 0) {
+    const int zero = 0;
+    if (cudaMemcpyToSymbol(g_status, &zero, sizeof(int)) != cudaSuccess) return MK_ERR_CUDA;
+  }
+  return h;
+}
+
 static int attn_fwd_impl(const void *q, const void *k, const void *v, void *o, float *lse, int B,
                          int Hq, int Hkv, int S, int D, int causal, float scale,
                          const int32_t *cu_seqlens, void *stream, int stall_first_slot) {
@@ -930,32 +940,5 @@ int mk_attn_fwd_stall_test(const void *q, const void *k, const void *v, void *o,
   return mk::attn_fwd_impl(q, k, v, o, lse, B, Hq, Hkv, S, D, causal, scale, cu_seqlens, stream, 1);
 }
 
-const char *mk_attn_error_string(int status) {
-  switch (status) {
-    case MK_OK: return "success";
-    case MK_ERR_INVALID_ARG: return "invalid argument";
-    case MK_ERR_UNSUPPORTED: return "unsupported head dimension (64 or 128)";
-    case MK_ERR_ALIGNMENT: return "pointer not 16-byte aligned";
-    case MK_ERR_CUDA: return "CUDA call failed";
-    case MK_ERR_TIMEOUT: return "kernel wait timed out";
-    case MK_ERR_SCRATCH_LIMIT: return "sizes need more scratch than the static decode array holds";
-    default: return "unknown status";
-  }
-}
-
-int mk_attn_check_status(void *stream) {
-  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  if (cudaStreamSynchronize(st) != cudaSuccess) return MK_ERR_CUDA;
-  int h = 0;
-  if (cudaMemcpyFromSymbol(&h, mk::g_status, sizeof(int)) != cudaSuccess) return MK_ERR_CUDA;
-  if (h != 0) {
-    const int zero = 0;
-    if (cudaMemcpyToSymbol(mk::g_status, &zero, sizeof(int)) != cudaSuccess) return MK_ERR_CUDA;
-  }
-  const int hd = mk::decode_take_status();
-  return h != 0 ? h : hd;
-}
-
-int mk_attn_version(void) { return 300; }
 
 }  // extern "C"

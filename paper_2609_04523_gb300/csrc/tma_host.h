@@ -40,7 +40,10 @@ inline bool encode_tokens_heads_dim(CUtensorMap *map, const void *base, uint64_t
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Reads and clears the decode kernels' device status word (defined with them).
+// Read and clear the device status word of each kernel family (each defined
+// with its kernels).
+int fwd_take_status();
+int bwd_take_status();
 int decode_take_status();
 
 }  // namespace mk

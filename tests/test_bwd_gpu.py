@@ -1,0 +1,123 @@
+"""Attention backward on the GPU against the fp64 oracle, through the C ABI.
+
+The GPU forward pass produces o and lse; the GPU backward pass then gives
+dq, dk, dv, which are compared element by element with the oracle's exact
+gradients of the forward definition.  Tolerance, from a rounding model of the
+kernel's arithmetic (P and dS rounded to bf16 as MMA operands, fp32
+accumulation, Delta from the bf16 o, bf16 outputs), which predicts a relative
+RMS error of about 2.4e-3 and a largest error of about 3.4e-3 of the largest
+gradient at these sizes: for each of dq, dk, dv, relative RMS <= 5e-3 and
+max |err| <= 1e-2 * max(max |ref|, 1e-3).  The floor covers gradients the
+mathematics makes exactly zero (one key: dq = dk = 0), where the kernel's
+Delta - dP cancellation leaves rounding residue near 1e-6."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_04523_gb300 import binding
+from paper_2609_04523_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+REL_RMS, MAX_REL = 5e-3, 1e-2
+ABS_FLOOR = 1e-3  # max-abs bound at least 1e-5, for gradients that are exactly zero
+
+
+def gpu_fwd_bwd(q, k, v, do, causal, scale, cu=None):
+    dev = torch.device("cuda")
+    qd, kd, vd, dod = (t.to(dev) for t in (q, k, v, do))
+    cud = None if cu is None else cu.to(dev)
+    o, lse = binding.attn_fwd(qd, kd, vd, causal=causal, scale=scale, cu_seqlens=cud)
+    dq = torch.full_like(qd, float("nan"))
+    dk = torch.full_like(kd, float("nan"))
+    dv = torch.full_like(vd, float("nan"))
+    binding.attn_bwd(qd, kd, vd, o, lse, dod, causal=causal, scale=scale, cu_seqlens=cud,
+                     dq=dq, dk=dk, dv=dv)
+    assert binding.mk_attn_check_status(torch.cuda.current_stream().cuda_stream) == binding.MK_OK
+    return dq.float().cpu().numpy(), dk.float().cpu().numpy(), dv.float().cpu().numpy()
+
+
+def compare(got, ref, what):
+    ref = np.asarray(ref, dtype=np.float64)
+    got = np.asarray(got, dtype=np.float64).reshape(ref.shape)
+    assert np.all(np.isfinite(got)), f"{what}: non-finite (unwritten) entries"
+    d = got - ref
+    scale = max(float(np.max(np.abs(ref))), ABS_FLOOR)
+    max_abs = float(np.max(np.abs(d)))
+    assert max_abs <= MAX_REL * scale, f"{what}: max_abs {max_abs:.3e} (max ref {scale:.3e})"
+    ref2 = float(np.sum(ref * ref))
+    if ref2 > 0.0:  # a gradient the mathematics makes zero has no relative error
+        rel = math.sqrt(float(np.sum(d * d)) / ref2)
+        assert rel <= REL_RMS, f"{what}: rel_rms {rel:.3e}"
+
+
+def check(q, k, v, do, causal, scale, cu=None, what=""):
+    dq, dk, dv = gpu_fwd_bwd(q, k, v, do, causal, scale, cu)
+    rq, rk, rv = oracle.attn_bwd(q, k, v, do, causal, scale,
+                                 cu_seqlens=None if cu is None else cu.numpy())
+    compare(dq, rq, f"{what} dq")
+    compare(dk, rk, f"{what} dk")
+    compare(dv, rv, f"{what} dv")
+
+
+@pytest.mark.parametrize("D", [64, 128])
+@pytest.mark.parametrize("causal", [True, False])
+@pytest.mark.parametrize("S", [1, 100, 128, 300, 513])
+def test_bwd_fixed_length(D, causal, S):
+    """Single partial tile, exact tiles and ragged tails; GQA group of 3."""
+    B, Hq, Hkv = 2, 6, 2
+    q, k, v, _ = W.make_qkv(B, Hq, Hkv, S, D, seed=800 + S + D + int(causal))
+    do = W.make_grad_out(q.shape, seed=800 + S + D)
+    check(q, k, v, do, causal, 1.0 / math.sqrt(D), what=f"S{S} D{D} causal={causal}")
+
+
+@pytest.mark.parametrize("G", [1, 4, 8])
+def test_bwd_group_sizes(G):
+    q, k, v, _ = W.make_qkv(1, 2 * G, 2, 640, 128, seed=850 + G)
+    do = W.make_grad_out(q.shape, seed=850 + G)
+    check(q, k, v, do, True, 1.0 / math.sqrt(128), what=f"G{G}")
+
+
+@pytest.mark.parametrize("causal", [True, False])
+@pytest.mark.parametrize("D", [64, 128])
+def test_bwd_varlen(causal, D):
+    """Packed sequences, including lengths below one tile and of one token."""
+    lens = [1, 130, 700, 5, 256, 383]
+    q, k, v, cu = W.make_qkv(0, 8, 2, 0, D, seed=870 + D + int(causal), lengths=lens)
+    do = W.make_grad_out(q.shape, seed=870 + D)
+    check(q, k, v, do, causal, 1.0 / math.sqrt(D), cu=cu, what=f"varlen D{D} causal={causal}")
+
+
+@pytest.mark.parametrize("scale", [-0.09, 0.0, 0.3])
+def test_bwd_scales(scale):
+    """Negative, zero and large scales (zero scale: dq = dk = 0)."""
+    q, k, v, _ = W.make_qkv(1, 4, 4, 260, 64, seed=890)
+    do = W.make_grad_out(q.shape, seed=890)
+    if scale == 0.0:
+        dq, dk, dv = gpu_fwd_bwd(q, k, v, do, True, 0.0)
+        assert np.all(dq == 0.0) and np.all(dk == 0.0)
+        _, _, rv = oracle.attn_bwd(q, k, v, do, True, 0.0)
+        compare(dv, rv, "scale 0 dv")
+        return
+    check(q, k, v, do, True, scale, what=f"scale {scale}")
+
+
+def test_bwd_deterministic():
+    """No atomics: two calls give bitwise identical gradients."""
+    q, k, v, _ = W.make_qkv(2, 8, 2, 777, 128, seed=900)
+    do = W.make_grad_out(q.shape, seed=900)
+    a = gpu_fwd_bwd(q, k, v, do, True, 0.088)
+    b = gpu_fwd_bwd(q, k, v, do, True, 0.088)
+    for x, y in zip(a, b):
+        assert np.array_equal(x, y)
+
+
+def test_bwd_causal_gqa_b4_s2048():
+    """The bench workload (causal GQA B=4, Hq=32, Hkv=8, S=2048, D=128), every
+    gradient element against the full oracle."""
+    inp = W.make_config_inputs(2)
+    do = W.make_grad_out(inp.q.shape, seed=inp.cfg.seed)
+    check(inp.q, inp.k, inp.v, do, True, inp.cfg.scale, what="B4 S2048")
