@@ -17,9 +17,14 @@ meet at a barrier around the timed region and rank 0 reports the maximum time.
 64 sequences of 1024-8192 cached tokens, Hq=32, Hkv=8, D=128, page_size=64)
 and reports HBM GB/s against the measured copy bandwidth.
 
+--workload backward times the backward pass (mk_attn_bwd: Delta, dK/dV and
+dQ kernels) on the same configs, in TFLOP/s of 2.5x the forward's FLOPs (the
+usual convention: five matmuls against the forward's two), and reports the
+dK/dV kernel, timed alone, against the bf16 tensor roofline.
+
 --impl reference times the fp64 CPU oracle on bounded row samples of the same
-workload (the whole step for decode; rank 0 only; other ranks exit without
-work).
+workload (the whole step for decode, one sequence for the backward pass;
+rank 0 only; other ranks exit without work).
 """
 from __future__ import annotations
 
@@ -38,10 +43,12 @@ sys.path.insert(0, ROOT)
 
 METRIC = "attention fwd TFLOP/s (causal FLOPs) and % of GB300 bf16 tensor peak"
 DECODE_METRIC = "paged decode step HBM GB/s (algorithmic bytes) and % of measured HBM copy bandwidth"
+BWD_METRIC = "attention bwd TFLOP/s (2.5x causal forward FLOPs) and % of GB300 bf16 tensor peak"
 NOMINAL_BF16_TFLOPS = 2250.0
 FLUSH_BYTES = 256 << 20
 KERNEL_SOURCES = ["paper_2609_04523_gb300/csrc/fmha_fwd.cu", "paper_2609_04523_gb300/csrc/ptx.cuh"]
 DECODE_SOURCES = ["paper_2609_04523_gb300/csrc/decode.cu", "paper_2609_04523_gb300/csrc/ptx.cuh"]
+BWD_SOURCES = ["paper_2609_04523_gb300/csrc/fmha_bwd.cu", "paper_2609_04523_gb300/csrc/ptx.cuh"]
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "ncu_traffic.json")
 BAD_REASONS = {"hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown"}
 
@@ -52,7 +59,7 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5])
-    ap.add_argument("--workload", default="prefill", choices=["prefill", "decode"],
+    ap.add_argument("--workload", default="prefill", choices=["prefill", "decode", "backward"],
                     help="prefill: the attention forward pass (--config); decode: one paged "
                          "decode step (the decode workload below)")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
@@ -653,6 +660,265 @@ def run_decode_reference(args, rank: int):
     }
 
 
+# ------------------------------------------------------------ backward pass
+
+def bwd_sample(inp):
+    """The first sequence of the workload, all heads: the oracle's backward
+    sample (its tasks are (sequence, key/value head) pairs)."""
+    c = inp.cfg
+    L = inp.lengths[0]
+    if c.varlen:
+        sl = slice(0, L)
+        return (inp.q[sl][None].contiguous(), inp.k[sl][None].contiguous(),
+                inp.v[sl][None].contiguous(), L)
+    return inp.q[:1].contiguous(), inp.k[:1].contiguous(), inp.v[:1].contiguous(), L
+
+
+def cpu_oracle_bwd(inp, do, prefix: int | None = None):
+    """Times the fp64 oracle's backward pass on the first sequence of the
+    workload (all heads), or on its first `prefix` tokens (itself a complete
+    problem when causal).  Returns (TFLOP/s by the 2.5x convention, threads
+    used, description, (dq, dk, dv) of the sample)."""
+    import oracle
+    from paper_2609_04523_gb300 import workloads as W
+    c = inp.cfg
+    q, k, v, L = bwd_sample(inp)
+    dos = do[:L][None].contiguous() if c.varlen else do[:1].contiguous()
+    if prefix is not None and prefix < L:
+        L = prefix
+        q, k, v, dos = (t[:, :L].contiguous() for t in (q, k, v, dos))
+    threads = min(oracle.default_threads(), c.Hkv)
+    t0 = time.perf_counter()
+    grads = oracle.attn_bwd(q, k, v, dos, c.causal, c.scale, n_threads=threads)
+    dt = time.perf_counter() - t0
+    fl = 2.5 * W.attn_flops([L], c.Hq, c.D, c.causal)
+    desc = (f"sequence 0 of the workload (first {L} tokens, all {c.Hq} query heads), "
+            f"{fl / 1e9:.1f} GFLOP by the 2.5x convention, {dt:.1f} s on {threads} threads "
+            f"(one per key/value head)")
+    return fl / dt / 1e12, threads, desc, grads
+
+
+def run_backward(args, rank: int, world: int, local_rank: int):
+    import numpy as np
+    import torch
+
+    from paper_2609_04523_gb300 import attn_bwd, attn_fwd, binding, mk_attn_check_status
+    from paper_2609_04523_gb300 import workloads as W
+    from paper_2609_04523_gb300.build import build_library
+
+    build_library()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    inp = W.make_config_inputs(args.config)
+    c = inp.cfg
+    fwd_flops = W.attn_flops(inp.lengths, c.Hq, c.D, c.causal)
+    flops = 2.5 * fwd_flops
+    do_h = W.make_grad_out(inp.q.shape, seed=c.seed)
+    q, k, v, do = inp.q.to(dev), inp.k.to(dev), inp.v.to(dev), do_h.to(dev)
+    cu = None if inp.cu_seqlens is None else inp.cu_seqlens.to(dev)
+    stream = torch.cuda.current_stream(dev)
+    o, lse = attn_fwd(q, k, v, c.causal, c.scale, cu, stream=stream)
+    dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+    T = sum(inp.lengths)
+    need = binding.mk_attn_bwd_workspace_bytes(1 if c.varlen else c.B, c.Hq,
+                                               T if c.varlen else c.S, c.varlen)
+    ws = torch.empty((need + 15) // 16 * 4, dtype=torch.float32, device=dev)
+    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    props = torch.cuda.get_device_properties(dev)
+    pci_bus_id = None
+    if hasattr(props, "pci_bus_id"):
+        pci_bus_id = "%08x:%02x:%02x.0" % (getattr(props, "pci_domain_id", 0), props.pci_bus_id,
+                                           getattr(props, "pci_device_id", 0))
+
+    def step(stages=binding.BWD_ALL):
+        attn_bwd(q, k, v, o, lse, do, c.causal, c.scale, cu, dq=dq, dk=dk, dv=dv, workspace=ws,
+                 stream=stream, stages=stages)
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize(dev)
+    if mk_attn_check_status(stream.cuda_stream) != 0:
+        raise RuntimeError("kernel reported a timeout during warm-up")
+
+    def timed(stages):
+        starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize(dev)
+        with ClockSampler(pci_bus_id, local_rank) as cs:
+            for i in range(args.steps):
+                flush.zero_()
+                starts[i].record(stream)
+                step(stages)
+                ends[i].record(stream)
+            torch.cuda.synchronize(dev)
+        if world > 1:
+            torch.distributed.barrier()
+        return [s_.elapsed_time(e_) for s_, e_ in zip(starts, ends)], cs.summary()
+
+    ms, clocks = timed(binding.BWD_ALL)
+    remeasured = False
+    if clocks_rejected(clocks):
+        ms, clocks = timed(binding.BWD_ALL)
+        remeasured = True
+    # Each kernel alone (Delta is already in the workspace), for the roofline.
+    ms_dkdv, _ = timed(binding.BWD_DKDV)
+    ms_dq, _ = timed(binding.BWD_DQ)
+    ms_delta, _ = timed(binding.BWD_DELTA)
+    if mk_attn_check_status(stream.cuda_stream) != 0:
+        raise RuntimeError("kernel reported a timeout in the timed region")
+    total_ms = max_over_ranks(sum(ms), world, dev)
+    ms_per_step = total_ms / args.steps
+    tflops_job = job_tflops(flops, args.steps, total_ms, world)
+    per_step_tflops = flops / (ms_per_step * 1e-3) / 1e12
+    t_dkdv = statistics.mean(ms_dkdv) * 1e-3
+    t_dq = statistics.mean(ms_dq) * 1e-3
+    dkdv_tflops = 2.0 * fwd_flops / t_dkdv / 1e12  # S^T, dP^T, dV, dK: four matmuls
+    dq_tflops = 1.5 * fwd_flops / t_dq / 1e12      # S, dP (recomputed), dQ: three matmuls
+
+    # End to end: pinned host q, k, v, o, lse, dO in; dq, dk, dv out.
+    o_h = torch.empty(o.shape, dtype=o.dtype).pin_memory()
+    l_h = torch.empty(lse.shape, dtype=lse.dtype).pin_memory()
+    o_h.copy_(o)
+    l_h.copy_(lse)
+    hosts_in = [inp.q.pin_memory(), inp.k.pin_memory(), inp.v.pin_memory(), o_h, l_h,
+                do_h.pin_memory()]
+    if inp.cu_seqlens is not None:
+        hosts_in.append(inp.cu_seqlens.pin_memory())
+    devs_in = [torch.empty_like(t, device=dev) for t in hosts_in]
+    hosts_out = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in (dq, dk, dv)]
+    h2d = sum(t.numel() * t.element_size() for t in hosts_in)
+    d2h = sum(t.numel() * t.element_size() for t in hosts_out)
+
+    def e2e_step():
+        for d_, h_ in zip(devs_in, hosts_in):
+            d_.copy_(h_, non_blocking=True)
+        cud = devs_in[6] if inp.cu_seqlens is not None else None
+        attn_bwd(devs_in[0], devs_in[1], devs_in[2], devs_in[3], devs_in[4], devs_in[5],
+                 c.causal, c.scale, cud, dq=dq, dk=dk, dv=dv, workspace=ws, stream=stream)
+        for h_, d_ in zip(hosts_out, (dq, dk, dv)):
+            h_.copy_(d_, non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        torch.distributed.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    e2e_tflops = job_tflops(flops, args.steps, e2e_ms, world)
+
+    if rank != 0:
+        return None
+    peaks, peak_src = measured_peaks()
+    peak = float(peaks["bf16_tflops"])
+    line = {
+        "metric": BWD_METRIC,
+        "value": round(tflops_job, 2),
+        "unit": "TFLOP/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 5),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,sigma^2) bf16 q, k, v and output gradient of the "
+                "workload's shape; o and lse from the GPU forward pass)",
+        "config": {
+            "workload": f"backward of {c.name}: {c.description}",
+            "config_index": c.index,
+            "flops_per_step_per_gpu": flops,
+            "flop_convention": "2.5 x the forward's 4*D*L^2 per sequence and head, halved when causal",
+            "pct_of_nominal_2250_tflops": round(100.0 * per_step_tflops / NOMINAL_BF16_TFLOPS, 2),
+            "kernel_ms": {"delta": round(statistics.mean(ms_delta), 5),
+                          "dkdv": round(t_dkdv * 1e3, 5), "dq": round(t_dq * 1e3, 5)},
+            "l2": "flushed before every timed step (256 MiB device write, outside the event pair)",
+            "timing": "CUDA events around each call (Delta, dK/dV and dQ kernels) on the launching "
+                      "stream; sum over steps; each kernel also timed alone the same way",
+            "parallelism": f"replicas x{world} (independent workloads per GPU)",
+        },
+        "roofline": {
+            "bound": "tensor",
+            "achieved": round(dkdv_tflops, 2),
+            "peak": peak,
+            "unit": "TFLOP/s",
+            "frac": round(dkdv_tflops / peak, 4),
+            "traffic": ncu_traffic("bwd_" + c.name, BWD_SOURCES),
+            "peak_source": f"{peak_src} bf16 burst (MEASURED_PEAKS.json bf16_tflops)",
+            "kernel": f"mk::bwd::bwd_kernel<{c.D}, false> (dK/dV: 4 matmuls, 2x forward FLOPs)",
+            "dq_kernel_tflops_executed": round(dq_tflops, 2),
+        },
+        "e2e": {"value": round(e2e_tflops, 2), "unit": "TFLOP/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": 3 * args.steps,
+        "clocks": clocks,
+    }
+    if remeasured:
+        line["clocks_note"] = "first timed region saw a rejected clock state; re-measured once"
+    if not args.no_cpu_baseline:
+        val, cores, desc, grads = cpu_oracle_bwd(inp, do_h)
+        line["cpu_baseline"] = {"value": round(val, 6), "unit": "TFLOP/s", "cores": cores,
+                                "kind": "oracle", "sample": desc}
+        L = inp.lengths[0]
+        got = [t.float().cpu().numpy() for t in (dq, dk, dv)]
+        got = [g[:L] if c.varlen else g[0] for g in got]
+        spot = {}
+        for name, g, r in zip(("dq", "dk", "dv"), got, grads):
+            r = r[0]
+            d = g - r
+            spot[name + "_max_abs"] = float(np.max(np.abs(d)))
+            spot[name + "_rel_rms"] = float(math.sqrt(np.sum(d * d) / np.sum(r * r)))
+        line["parity_spot_check"] = dict(rows=f"sequence 0, all heads ({L} tokens)", **spot)
+    return line
+
+
+def run_backward_reference(args, rank: int):
+    """The oracle's backward pass, as it stands, on the first sequence of the
+    workload each step."""
+    if rank != 0:
+        return None
+    from paper_2609_04523_gb300 import workloads as W
+    inp = W.make_config_inputs(args.config)
+    c = inp.cfg
+    do_h = W.make_grad_out(inp.q.shape, seed=c.seed)
+    # A causal prefix of sequence 0 sized so that the whole run stays within a
+    # few minutes: the oracle's time grows with the square of the prefix.
+    budget = max(1.0, min(10.0, 150.0 / max(1, args.steps + args.warmup)))
+    t0 = time.perf_counter()
+    cpu_oracle_bwd(inp, do_h, prefix=256)
+    t256 = max(time.perf_counter() - t0, 1e-3)
+    prefix = int(256 * math.sqrt(budget / t256)) if c.causal else None
+    vals, cores, desc = [], None, None
+    for i in range(args.warmup + args.steps):
+        val, cores, desc, _ = cpu_oracle_bwd(inp, do_h, prefix=prefix)
+        if i >= args.warmup:
+            vals.append(val)
+    value = statistics.median(vals)
+    return {
+        "impl": "reference", "metric": BWD_METRIC, "value": round(value, 6), "unit": "TFLOP/s",
+        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": None,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded N(0,sigma^2) bf16 q, k, v and output gradient)",
+        "config": {"workload": f"backward of {c.name}: {c.description}", "config_index": c.index,
+                   "note": "the fp64 CPU oracle, as it stands, on a causal prefix of the first "
+                           "sequence per step"},
+        "cpu_baseline": {"value": round(value, 6), "unit": "TFLOP/s", "cores": cores,
+                         "kind": "oracle", "sample": f"per step: {desc}"},
+        "e2e": {"value": round(value, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+        "gpu_launches": 0,
+    }
+
+
 # ----------------------------------------------------------- reference arm
 
 def run_reference(args, rank: int):
@@ -701,8 +967,12 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
-        line = run_decode_reference(args, rank) if args.workload == "decode" else \
-            run_reference(args, rank)
+        if args.workload == "decode":
+            line = run_decode_reference(args, rank)
+        elif args.workload == "backward":
+            line = run_backward_reference(args, rank)
+        else:
+            line = run_reference(args, rank)
         if line is not None:
             print(json.dumps(line), flush=True)
         return
@@ -711,8 +981,12 @@ def main():
         torch.cuda.set_device(local_rank)
         torch.distributed.init_process_group("nccl")
     try:
-        line = run_decode(args, rank, world, local_rank) if args.workload == "decode" else \
-            run_ours(args, rank, world, local_rank)
+        if args.workload == "decode":
+            line = run_decode(args, rank, world, local_rank)
+        elif args.workload == "backward":
+            line = run_backward(args, rank, world, local_rank)
+        else:
+            line = run_ours(args, rank, world, local_rank)
     finally:
         if world > 1:
             import torch

@@ -145,6 +145,27 @@ MK_API int mk_attn_bwd(const void *q, const void *k, const void *v, const void *
                        const int32_t *cu_seqlens, void *workspace, int64_t workspace_bytes,
                        void *stream);
 
+/* Stages of the backward pass, for mk_attn_bwd_stages. */
+#define MK_BWD_DELTA 1 /* Delta_i = dO_i . o_i into the workspace */
+#define MK_BWD_DKDV 2  /* dk and dv (reads Delta from the workspace) */
+#define MK_BWD_DQ 4    /* dq (reads Delta from the workspace) */
+#define MK_BWD_ALL 7
+
+/*
+ * mk_attn_bwd_stages -- mk_attn_bwd, enqueuing only the stages in `stages`
+ * (a nonzero OR of the MK_BWD_* flags), in the order Delta, dK/dV, dQ.
+ * Arguments, checks and errors are those of mk_attn_bwd.  MK_BWD_DKDV and
+ * MK_BWD_DQ read the Delta that an earlier MK_BWD_DELTA stage wrote into the
+ * same workspace for the same o and dO; once it is there, the two are
+ * independent of each other (e.g. on two streams, ordered after Delta by the
+ * caller).  Outputs of stages not enqueued are left untouched.
+ */
+MK_API int mk_attn_bwd_stages(const void *q, const void *k, const void *v, const void *o,
+                              const float *lse, const void *dO, void *dq, void *dk, void *dv,
+                              int B, int Hq, int Hkv, int S, int D, int causal, float scale,
+                              const int32_t *cu_seqlens, void *workspace,
+                              int64_t workspace_bytes, int stages, void *stream);
+
 /*
  * mk_attn_decode_workspace_bytes -- bytes of device workspace that
  * mk_attn_decode_paged needs for these sizes on the current device (0: none),

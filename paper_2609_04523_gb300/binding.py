@@ -21,11 +21,15 @@ MK_ERR_CUDA = -4
 MK_ERR_TIMEOUT = -5
 MK_ERR_SCRATCH_LIMIT = -6
 
+# Backward-pass stages (MK_BWD_* in include/mk_attn.h).
+BWD_DELTA, BWD_DKDV, BWD_DQ, BWD_ALL = 1, 2, 4, 7
+
 # Bytes of the library's own decode scratch array (MK_ATTN_DECODE_STATIC_SCRATCH_BYTES).
 DECODE_STATIC_SCRATCH_BYTES = 8 * 1024 * 1024
 
 # Symbols declared in include/mk_attn.h.
 EXPORTED = ("mk_attn_fwd", "mk_attn_fwd_stall_test", "mk_attn_bwd_workspace_bytes", "mk_attn_bwd",
+            "mk_attn_bwd_stages",
             "mk_attn_decode_workspace_bytes",
             "mk_attn_decode_paged", "mk_attn_decode_paged_noalloc", "mk_attn_error_string",
             "mk_attn_check_status", "mk_attn_version")
@@ -66,6 +70,8 @@ def load_library() -> ctypes.CDLL:
             lib.mk_attn_bwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, i, i, i, i, i, i,
                                         ctypes.c_float, vp, vp, i64, vp]
             lib.mk_attn_bwd.restype = i
+            lib.mk_attn_bwd_stages.argtypes = lib.mk_attn_bwd.argtypes[:-1] + [i, vp]
+            lib.mk_attn_bwd_stages.restype = i
             lib.mk_attn_decode_workspace_bytes.argtypes = [i, i, i, i, i, i]
             lib.mk_attn_decode_workspace_bytes.restype = i64
             lib.mk_attn_decode_paged.argtypes = [vp, vp, vp, vp, vp, vp, vp, i, i, i, i, i, i, i,
@@ -180,14 +186,27 @@ def mk_attn_bwd(q: int, k: int, v: int, o: int, lse: int, do: int, dq: int, dk: 
                                       int(workspace_bytes), stream)
 
 
+def mk_attn_bwd_stages(q: int, k: int, v: int, o: int, lse: int, do: int, dq: int, dk: int,
+                       dv: int, B: int, Hq: int, Hkv: int, S: int, D: int, causal: int,
+                       scale: float, cu_seqlens: int | None, workspace: int | None,
+                       workspace_bytes: int, stages: int, stream: int | None) -> int:
+    """Raw C-ABI call of selected backward stages (BWD_* flags)."""
+    return load_library().mk_attn_bwd_stages(q, k, v, o, lse, do, dq, dk, dv, B, Hq, Hkv, S, D,
+                                             int(causal), float(scale), cu_seqlens, workspace,
+                                             int(workspace_bytes), int(stages), stream)
+
+
 def attn_bwd(q, k, v, o, lse, do, causal: bool = True, scale: float | None = None,
-             cu_seqlens=None, dq=None, dk=None, dv=None, workspace=None, stream=None):
+             cu_seqlens=None, dq=None, dk=None, dv=None, workspace=None, stream=None,
+             stages: int = BWD_ALL):
     """Attention backward on CUDA tensors through mk_attn_bwd.
 
     q, k, v, causal, scale, cu_seqlens as for attn_fwd; o, lse its outputs;
     do: bf16 gradient of o (layout of q).  Returns (dq, dk, dv), bf16, the
-    layouts of q, k, v.  PyTorch only allocates the outputs and the fp32
-    workspace and provides the stream."""
+    layouts of q, k, v.  `stages` (BWD_* flags) enqueues only some of the three
+    kernels; dK/dV and dQ need the Delta an earlier call wrote into the same
+    `workspace`.  PyTorch only allocates the outputs and the fp32 workspace and
+    provides the stream."""
     import torch
     for name, t in (("q", q), ("k", k), ("v", v), ("o", o), ("do", do)):
         if not t.is_cuda or t.dtype != torch.bfloat16 or not t.is_contiguous():
@@ -227,10 +246,12 @@ def attn_bwd(q, k, v, o, lse, do, causal: bool = True, scale: float | None = Non
         workspace = torch.empty((need + 15) // 16 * 4, dtype=torch.float32, device=q.device)
     if stream is None:
         stream = torch.cuda.current_stream(q.device)
-    _check(mk_attn_bwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), o.data_ptr(), lse.data_ptr(),
-                       do.data_ptr(), dq.data_ptr(), dk.data_ptr(), dv.data_ptr(), B, Hq, Hkv, S,
-                       D, int(bool(causal)), float(scale), cu_ptr, workspace.data_ptr(),
-                       workspace.numel() * workspace.element_size(), stream.cuda_stream))
+    _check(mk_attn_bwd_stages(q.data_ptr(), k.data_ptr(), v.data_ptr(), o.data_ptr(),
+                              lse.data_ptr(), do.data_ptr(), dq.data_ptr(), dk.data_ptr(),
+                              dv.data_ptr(), B, Hq, Hkv, S, D, int(bool(causal)), float(scale),
+                              cu_ptr, workspace.data_ptr(),
+                              workspace.numel() * workspace.element_size(), int(stages),
+                              stream.cuda_stream))
     return dq, dk, dv
 
 

@@ -73,24 +73,36 @@ constexpr float kLog2e = 1.4426950408889634f;
 
 __device__ int g_status = 0;  // MK_ERR_TIMEOUT once a wait ran out
 
-template <int D>
+// Ring depths: Y1 is the load on the critical path (its slot frees only when
+// the last MMA of an iteration has read it), so it gets the deeper ring where
+// shared memory allows: at D = 128 the dQ kernel has room for three Y1
+// stages, the dK/dV kernel (which also stages lse / Delta vectors per Y1
+// stage) for two.
+template <int D, bool DQ>
 struct Cfg {
   static_assert(D == 64 || D == 128, "head dimension 64 or 128");
-  static constexpr int kStages = (D == 128) ? 2 : 4;
+  static constexpr int kStages1 = (D == 128) ? (DQ ? 3 : 2) : 4;
+  static constexpr int kStages2 = (D == 128) ? 2 : 4;
   static constexpr int kHalves = D / kBoxCols;
   static constexpr int kTileBytes = kTile * D * 2;
   static constexpr int kOffX1 = 0;               // K (dK/dV) or Q (dQ)
   static constexpr int kOffX2 = kTileBytes;      // V (dK/dV) or dO (dQ)
-  static constexpr int kOffY = 2 * kTileBytes;   // slot s: Y1 at + 2 s T, Y2 at + (2 s + 1) T
-  static constexpr int kOffVec = kOffY + kStages * 2 * kTileBytes;  // [stage][lse2 | delta][128]
-  static constexpr int kOffCtl = kOffVec + kStages * 2 * kTile * 4;
+  static constexpr int kOffY1 = 2 * kTileBytes;  // Y1 ring: Q (dK/dV) or K (dQ)
+  static constexpr int kOffY2 = kOffY1 + kStages1 * kTileBytes;  // Y2 ring: dO or V
+  static constexpr int kOffVec = kOffY2 + kStages2 * kTileBytes;  // dK/dV: [stage][lse2 | delta][128]
+  static constexpr int kOffCtl = kOffVec + (DQ ? 0 : kStages1 * 2 * kTile * 4);
   static constexpr int kSmemBytes = kOffCtl + 256 + 1024;
+  static_assert(kSmemBytes <= 232448, "shared memory per CTA");
 };
 
+// Streamed operands have a ring each: Y1 (Q for dK/dV, K for dQ) and Y2 (dO,
+// or V).  Y2's last reader (dV, or dP) finishes long before Y1's (dK, or dQ),
+// so separate barriers let the producer refill Y2 early and leave only Y1's
+// load on the critical path.
 struct Ctl {
   uint64_t fixed_full, fixed_empty;
-  uint64_t y_full[4], y_empty[4];
-  uint64_t s_full, dp_full, p_full, ds_full, acc_full, mma_drained;
+  uint64_t y1_full[4], y1_empty[4], y2_full[4], y2_empty[4];
+  uint64_t s_full, dp_full, p_full, dp_free, ds_full, acc_full, mma_drained;
   uint32_t tmem_base;
   int abort;
 };
@@ -212,8 +224,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     bwd_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
                const Params p) {
-  using C = Cfg<D>;
-  constexpr int NS = C::kStages;
+  using C = Cfg<D, DQ>;
+  constexpr int NS1 = C::kStages1;
+  constexpr int NS2 = C::kStages2;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = smem_addr(smem_raw);
   uint8_t *smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);
@@ -224,15 +237,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     mbar_init(&ctl->fixed_full, 1);
     mbar_init(&ctl->fixed_empty, 1);
-    for (int s = 0; s < NS; ++s) {
-      // dK/dV: the TMA bytes plus one arrival per producer lane for the
-      // lse / Delta vectors the lanes write.
-      mbar_init(&ctl->y_full[s], DQ ? 1 : 33);
-      mbar_init(&ctl->y_empty[s], 1);
+    for (int s = 0; s < NS1; ++s) {
+      // Y1 of dK/dV: the TMA bytes plus one arrival per producer lane for
+      // the lse / Delta vectors the lanes write.
+      mbar_init(&ctl->y1_full[s], DQ ? 1 : 33);
+      mbar_init(&ctl->y1_empty[s], 1);
+    }
+    for (int s = 0; s < NS2; ++s) {
+      mbar_init(&ctl->y2_full[s], 1);
+      mbar_init(&ctl->y2_empty[s], 1);
     }
     mbar_init(&ctl->s_full, 1);
     mbar_init(&ctl->dp_full, 1);
     mbar_init(&ctl->p_full, kEwThreads);
+    mbar_init(&ctl->dp_free, kEwThreads);
     mbar_init(&ctl->ds_full, kEwThreads);
     mbar_init(&ctl->acc_full, 1);
     mbar_init(&ctl->mma_drained, 1);
@@ -289,65 +307,82 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       ++n_unit;
       const int nq = tiles_of(w.len) - first_q;
-      for (int n = 0; n < N; ++n) {
-        const int s = it % NS;
-        ok = mbar_wait_all(&ctl->y_empty[s], ((it / NS) & 1) ^ 1, abort);
-        if (!ok) break;
-        uint8_t *y1 = smem + C::kOffY + 2 * s * C::kTileBytes;
-        uint8_t *y2 = y1 + C::kTileBytes;
-        if constexpr (DQ) {
-          if (elect_one()) {
-            mbar_arrive_expect_tx(&ctl->y_full[s], 2 * C::kTileBytes);
-            const int row0 = w.seq_start + n * kTile;
-            const int g = w.head / p.G;
-            load_tile(y1, &tm_k, &ctl->y_full[s], g, row0);
-            load_tile(y2, &tm_v, &ctl->y_full[s], g, row0);
-          }
-        } else {
-          const int h = w.head * p.G + n / nq;
-          const int qt = first_q + n % nq;
-          // lse in base 2 and Delta of the tile's 128 query positions;
-          // positions past the sequence end get lse2 = +inf (P = 0) and
-          // Delta = 0, so they contribute nothing.
-          float *lv = vec + s * 2 * kTile;
+      // dK/dV: lse in base 2 and Delta of the 128 query positions of streamed
+      // tile n, 4 per lane, loaded one tile ahead so that their latency
+      // overlaps the wait for a free slot; positions past the sequence end get
+      // lse2 = +inf (P = 0) and Delta = 0, so they contribute nothing.
+      float l2v[kTile / 32], dlv[kTile / 32];
+      auto fetch_vec = [&](int n) {
+        const int h = w.head * p.G + n / nq;
+        const int qt = first_q + n % nq;
 #pragma unroll
-          for (int e = 0; e < kTile / 32; ++e) {
-            const int pos = qt * kTile + e * 32 + lane;
-            float l2 = INFINITY, dl = 0.f;
-            if (pos < w.len) {
-              const int64_t ri = row_index(p, w, h, pos);
-              l2 = p.lse[ri] * kLog2e;
-              dl = p.delta[ri];
-            }
-            lv[e * 32 + lane] = l2;
-            lv[kTile + e * 32 + lane] = dl;
+        for (int e = 0; e < kTile / 32; ++e) {
+          const int pos = qt * kTile + e * 32 + lane;
+          l2v[e] = INFINITY;
+          dlv[e] = 0.f;
+          if (pos < w.len) {
+            const int64_t ri = row_index(p, w, h, pos);
+            l2v[e] = p.lse[ri] * kLog2e;
+            dlv[e] = p.delta[ri];
           }
-          __syncwarp();
-          if (elect_one()) {
-            mbar_arrive_expect_tx(&ctl->y_full[s], 2 * C::kTileBytes);
-            const int row0 = w.seq_start + qt * kTile;
-            load_tile(y1, &tm_q, &ctl->y_full[s], h, row0);
-            load_tile(y2, &tm_do, &ctl->y_full[s], h, row0);
-          }
-          __syncwarp();
-          mbar_arrive(&ctl->y_full[s]);  // every lane: its vector writes are released
+        }
+      };
+      if constexpr (!DQ) fetch_vec(0);
+      for (int n = 0; n < N; ++n) {
+        const int s1 = it % NS1, s2 = it % NS2;
+        uint8_t *y1 = smem + C::kOffY1 + s1 * C::kTileBytes;
+        uint8_t *y2 = smem + C::kOffY2 + s2 * C::kTileBytes;
+        // Head and token row of the streamed tiles: dQ streams the key tiles
+        // of the query head's key/value head; dK/dV streams the query tiles
+        // of each head of the group.
+        const int head = DQ ? w.head / p.G : w.head * p.G + n / nq;
+        const int row0 = w.seq_start + (DQ ? n : first_q + n % nq) * kTile;
+        // Y1 first: S needs it a whole elementwise phase before dP needs Y2.
+        ok = mbar_wait_all(&ctl->y1_empty[s1], ((it / NS1) & 1) ^ 1, abort);
+        if (!ok) break;
+        if (elect_one()) {
+          mbar_arrive_expect_tx(&ctl->y1_full[s1], C::kTileBytes);
+          load_tile(y1, DQ ? &tm_k : &tm_q, &ctl->y1_full[s1], head, row0);
         }
         __syncwarp();
+        if constexpr (!DQ) {
+          float *lv = vec + s1 * 2 * kTile;
+#pragma unroll
+          for (int e = 0; e < kTile / 32; ++e) {
+            lv[e * 32 + lane] = l2v[e];
+            lv[kTile + e * 32 + lane] = dlv[e];
+          }
+          mbar_arrive(&ctl->y1_full[s1]);  // every lane: its vector writes are released
+        }
+        ok = mbar_wait_all(&ctl->y2_empty[s2], ((it / NS2) & 1) ^ 1, abort);
+        if (!ok) break;
+        if (elect_one()) {
+          mbar_arrive_expect_tx(&ctl->y2_full[s2], C::kTileBytes);
+          load_tile(y2, DQ ? &tm_v : &tm_do, &ctl->y2_full[s2], head, row0);
+        }
+        __syncwarp();
+        if constexpr (!DQ) {
+          if (n + 1 < N) fetch_vec(n + 1);
+        }
         ++it;
       }
     }
     // Teardown: the loads issued land before the CTA exits.
     if (n_unit > 0) drain_wait(&ctl->fixed_full, (n_unit - 1) & 1);
-    for (uint32_t n = (it > (uint32_t)NS ? it - NS : 0); n < it; ++n)
-      drain_wait(&ctl->y_full[n % NS], (n / NS) & 1);
+    for (uint32_t n = (it > (uint32_t)NS1 ? it - NS1 : 0); n < it; ++n)
+      drain_wait(&ctl->y1_full[n % NS1], (n / NS1) & 1);
+    for (uint32_t n = (it > (uint32_t)NS2 ? it - NS2 : 0); n < it; ++n)
+      drain_wait(&ctl->y2_full[n % NS2], (n / NS2) & 1);
   } else if (warp == kMmaWarp) {
     // ---------------------------------------------------------- MMA issuer
     constexpr uint32_t idesc_ss = idesc_bf16_f32(kTile, kTile, false, false);
     constexpr uint32_t idesc_ts = idesc_bf16_f32(kTile, D, false, true);
     constexpr uint32_t kLbo = (D > kBoxCols) ? kBoxBytes : 1024;
     const uint32_t sX1 = smem_addr(smem + C::kOffX1), sX2 = smem_addr(smem + C::kOffX2);
-    const uint32_t sY = smem_addr(smem + C::kOffY);
-    constexpr uint32_t kColAcc2 = DQ ? kColAcc : kColAcc + D;
+    const uint32_t sY1 = smem_addr(smem + C::kOffY1), sY2 = smem_addr(smem + C::kOffY2);
+    // dQ: dS(i) (bf16, 64 columns: keys 0..63 from warpgroup 0, 64..127 from
+    // warpgroup 1) goes to buffer i % 2 after the dQ accumulator.
+    constexpr uint32_t kColDs = kColAcc + D;
     uint32_t n_unit = 0, it = 0, n_p = 0, n_ds = 0;
     bool ok = true;
     // D[tmem col] = X[smem] Y[smem]^T, both K-major (head dim contiguous).
@@ -362,12 +397,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     };
     // acc[tmem col] (+)= A[tmem a_col] Y[smem], Y MN-major (128 rows x D):
     // the 128-wide contraction runs over the rows of Y; its bf16 A operand
-    // sits in columns a_col + 0..31 (rows 0..63 of Y) and a_col + 64..95.
-    auto issue_acc = [&](uint32_t col, uint32_t a_col, uint32_t y_addr, bool accumulate) {
+    // sits in columns a_col + 0..31 (rows 0..63 of Y) and a_col + 32 + gap ..
+    // gap: 32 when the two 32-column halves sit in place in S / dP (columns
+    // a_col + 0..31 and + 64..95), 0 for a packed 64-column dS buffer.
+    auto issue_acc = [&](uint32_t col, uint32_t a_col, uint32_t gap, uint32_t y_addr,
+                         bool accumulate) {
       const uint64_t b0 = sdesc_sw128(y_addr, kLbo, 1024);
 #pragma unroll
       for (int kk = 0; kk < kTile / 16; ++kk) {
-        const uint32_t a = tmem + a_col + kk * 8 + (kk >= 4 ? 32 : 0);
+        const uint32_t a = tmem + a_col + kk * 8 + (kk >= 4 ? gap : 0);
         umma_ts(tmem + col, a, b0 + (uint64_t)(kk * 128), idesc_ts,
                 (accumulate || kk > 0) ? 1u : 0u);
       }
@@ -382,31 +420,42 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = mbar_wait_all(&ctl->fixed_full, n_unit & 1, abort);
       if (!ok) break;
       const uint32_t it0 = it;
-      auto y1_of = [&](uint32_t i) { return sY + 2 * (i % NS) * C::kTileBytes; };
-      ok = mbar_wait_all(&ctl->y_full[it0 % NS], (it0 / NS) & 1, abort);
+      auto y1_of = [&](uint32_t i) { return sY1 + (i % NS1) * C::kTileBytes; };
+      auto y2_of = [&](uint32_t i) { return sY2 + (i % NS2) * C::kTileBytes; };
+      ok = mbar_wait_all(&ctl->y1_full[it0 % NS1], (it0 / NS1) & 1, abort);
       if (!ok) break;
       tc_fence_after_sync();
       if (elect_one()) {
         issue_xy(kColS, sX1, y1_of(it0));
         umma_commit(&ctl->s_full);
-        issue_xy(kColP, sX2, y1_of(it0) + C::kTileBytes);
+      }
+      __syncwarp();
+      ok = mbar_wait_all(&ctl->y2_full[it0 % NS2], (it0 / NS2) & 1, abort);
+      if (!ok) break;
+      tc_fence_after_sync();
+      if (elect_one()) {
+        issue_xy(kColP, sX2, y2_of(it0));
         umma_commit(&ctl->dp_full);
+        if constexpr (DQ) umma_commit(&ctl->y2_empty[it0 % NS2]);  // V read by dP only
         if (N == 1) umma_commit(&ctl->fixed_empty);
       }
       __syncwarp();
       for (int n = 0; ok && n < N; ++n) {
         const uint32_t i = it0 + n;
+        const bool more = n + 1 < N;
         ok = mbar_wait_all(&ctl->p_full, n_p & 1, abort);
         ++n_p;
         if (!ok) break;
         tc_fence_after_sync();
         if constexpr (!DQ) {
-          if (elect_one()) issue_acc(kColAcc, kColS, y1_of(i) + C::kTileBytes, n > 0);  // dV += P dO
+          if (elect_one()) {
+            issue_acc(kColAcc, kColS, 32, y2_of(i), n > 0);  // dV += P dO
+            umma_commit(&ctl->y2_empty[i % NS2]);  // dO(n) no longer read
+          }
           __syncwarp();
         }
-        const bool more = n + 1 < N;
         if (more) {
-          ok = mbar_wait_all(&ctl->y_full[(i + 1) % NS], ((i + 1) / NS) & 1, abort);
+          ok = mbar_wait_all(&ctl->y1_full[(i + 1) % NS1], ((i + 1) / NS1) & 1, abort);
           if (!ok) break;
           tc_fence_after_sync();
           if (elect_one()) {
@@ -415,20 +464,43 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           __syncwarp();
         }
+        if constexpr (DQ) {
+          // dP(n) has been read into registers and dS(n) goes to its own
+          // buffer, so dP(n+1) need not wait for dQ(n).
+          ok = mbar_wait_all(&ctl->dp_free, (n_ds & 1), abort);
+          if (!ok) break;
+          if (more) {
+            ok = mbar_wait_all(&ctl->y2_full[(i + 1) % NS2], ((i + 1) / NS2) & 1, abort);
+            if (!ok) break;
+            tc_fence_after_sync();
+            if (elect_one()) {
+              issue_xy(kColP, sX2, y2_of(i + 1));
+              umma_commit(&ctl->dp_full);
+              umma_commit(&ctl->y2_empty[(i + 1) % NS2]);  // V read by dP only
+              if (n + 2 == N) umma_commit(&ctl->fixed_empty);
+            }
+            __syncwarp();
+          }
+        }
         ok = mbar_wait_all(&ctl->ds_full, n_ds & 1, abort);
         ++n_ds;
         if (!ok) break;
+        if (!DQ && more) ok = mbar_wait_all(&ctl->y2_full[(i + 1) % NS2], ((i + 1) / NS2) & 1, abort);
+        if (!ok) break;
         tc_fence_after_sync();
         if (elect_one()) {
-          issue_acc(kColAcc2, kColP, y1_of(i), n > 0);  // dK += dS Q, or dQ += dS K
-          umma_commit(&ctl->y_empty[i % NS]);
-          if (more) {
-            issue_xy(kColP, sX2, y1_of(i + 1) + C::kTileBytes);
+          if constexpr (DQ) {
+            issue_acc(kColAcc, kColDs + (i & 1) * 64, 0, y1_of(i), n > 0);  // dQ += dS K
+          } else {
+            issue_acc(kColAcc + D, kColP, 32, y1_of(i), n > 0);  // dK += dS Q
+          }
+          umma_commit(&ctl->y1_empty[i % NS1]);
+          if (!DQ && more) {
+            issue_xy(kColP, sX2, y2_of(i + 1));
             umma_commit(&ctl->dp_full);
             if (n + 2 == N) umma_commit(&ctl->fixed_empty);
-          } else {
-            umma_commit(&ctl->acc_full);
           }
+          if (!more) umma_commit(&ctl->acc_full);
         }
         __syncwarp();
       }
@@ -448,6 +520,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t n_unit = 0, it = 0, n_s = 0;
     bool ok = true;
     constexpr uint32_t kColAcc2 = DQ ? kColAcc : kColAcc + D;
+    static_assert(!DQ || kColAcc + D + 128 <= kTmemCols, "dS buffers");
     for (int k = 0; ok && k * (int)gridDim.x < p.n_units; ++k) {
       const int u = unit_of_round(k);
       if (u >= p.n_units) continue;
@@ -483,8 +556,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int c = 0; c < 64; ++c) x[c] = __uint_as_float(raw[c / 32][c % 32]);
         }
         // P = 2^(s * scale * log2 e - lse2), hidden pairs 0.
-        const float *lv = vec + (i % NS) * 2 * kTile;
+        const float *lv = vec + (i % NS1) * 2 * kTile;
         if constexpr (DQ) {
+          // S(n) is in registers: S(n+1) may overwrite it.
+          tc_fence_before_sync();
+          mbar_arrive(&ctl->p_full);
           const int kpos0 = n * kTile + col0;  // key position of column 0 of this half
           const int lim = p.causal ? min(w.len, qpos + 1) : w.len;  // keys [0, lim)
           const bool mask = kpos0 + 64 > lim;
@@ -497,7 +573,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           // The producer lanes wrote this slot's vectors before arriving on
           // its full barrier; that phase has completed (the MMA waited for it
           // before S) and cannot advance before this iteration ends.
-          ok = mbar_wait_all(&ctl->y_full[i % NS], (i / NS) & 1, abort);
+          ok = mbar_wait_all(&ctl->y1_full[i % NS1], (i / NS1) & 1, abort);
           if (!ok) break;
           const int qt = first_q + n % nq;
           const bool diag = p.causal && qt == w.tile;  // key row > query column hidden
@@ -519,9 +595,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int c = 0; c < 32; ++c) pk[c] = pack_bf16x2(x[2 * c], x[2 * c + 1]);
           tmem_st_32x32b_x32(t_row + kColS + col0, pk);
           tmem_st_wait();
+          tc_fence_before_sync();
+          mbar_arrive(&ctl->p_full);
         }
-        tc_fence_before_sync();
-        mbar_arrive(&ctl->p_full);
         ok = mbar_wait_all(&ctl->dp_full, n_s & 1, abort);
         ++n_s;
         if (!ok) break;
@@ -533,22 +609,28 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_ld_wait();
           reg_fence(raw[0]);
           reg_fence(raw[1]);
+          if constexpr (DQ) {  // dP(n) is in registers: dP(n+1) may overwrite it
+            tc_fence_before_sync();
+            mbar_arrive(&ctl->dp_free);
+          }
           uint32_t pk[32];
 #pragma unroll
-          for (int c = 0; c < 64; c += 2) {
-            float d0, d1;
+          for (int c = 0; c < 64; c += 4) {
+            float4 d4;
             if constexpr (DQ) {
-              d0 = row_dl;
-              d1 = row_dl;
+              d4 = make_float4(row_dl, row_dl, row_dl, row_dl);
             } else {
-              d0 = lv[kTile + col0 + c];
-              d1 = lv[kTile + col0 + c + 1];
+              d4 = *reinterpret_cast<const float4 *>(lv + kTile + col0 + c);
             }
-            const float ds0 = x[c] * (__uint_as_float(raw[c / 32][c % 32]) - d0);
-            const float ds1 = x[c + 1] * (__uint_as_float(raw[c / 32][c % 32 + 1]) - d1);
+            const float ds0 = x[c] * (__uint_as_float(raw[c / 32][c % 32]) - d4.x);
+            const float ds1 = x[c + 1] * (__uint_as_float(raw[c / 32][c % 32 + 1]) - d4.y);
+            const float ds2 = x[c + 2] * (__uint_as_float(raw[c / 32][c % 32 + 2]) - d4.z);
+            const float ds3 = x[c + 3] * (__uint_as_float(raw[c / 32][c % 32 + 3]) - d4.w);
             pk[c / 2] = pack_bf16x2(ds0, ds1);
+            pk[c / 2 + 1] = pack_bf16x2(ds2, ds3);
           }
-          tmem_st_32x32b_x32(t_row + kColP + col0, pk);
+          // dK/dV: dS^T in place of dP^T; dQ: dS into buffer i % 2.
+          tmem_st_32x32b_x32(t_row + (DQ ? kColAcc + D + (i & 1) * 64 + wg * 32 : kColP + col0), pk);
           tmem_st_wait();
         }
         tc_fence_before_sync();
@@ -647,12 +729,12 @@ static void kernel_setup(DeviceInfo &di) {
   const int vi = (D == 128 ? 2 : 0) + (DQ ? 1 : 0);
   di.attr_err[vi] = cudaFuncSetAttribute(bwd_kernel<D, DQ>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         Cfg<D>::kSmemBytes);
+                                         Cfg<D, DQ>::kSmemBytes);
 }
 
 template <int D>
 static int launch(const void *q, const void *k, const void *v, const void *o, const void *dO,
-                  Params p, int64_t tokens, cudaStream_t st) {
+                  Params p, int64_t tokens, int stages, cudaStream_t st) {
   CUtensorMap tq, tk, tv, tdo;
   if (!encode_tokens_heads_dim(&tq, q, tokens, p.Hq, D, kTile) ||
       !encode_tokens_heads_dim(&tk, k, tokens, p.Hkv, D, kTile) ||
@@ -674,22 +756,29 @@ static int launch(const void *q, const void *k, const void *v, const void *o, co
   if (di.sm_count <= 0 || di.attr_err[v0] != cudaSuccess || di.attr_err[v0 + 1] != cudaSuccess)
     return MK_ERR_CUDA;
   const int64_t rows = tokens * p.Hq;
-  delta_kernel<D><<<(unsigned)((rows * 16 + 255) / 256), 256, 0, st>>>(
-      reinterpret_cast<const uint16_t *>(o), reinterpret_cast<const uint16_t *>(dO),
-      const_cast<float *>(p.delta), rows, p.Hq, p.S, p.varlen);
-  if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
+  if (stages & 1) {
+    delta_kernel<D><<<(unsigned)((rows * 16 + 255) / 256), 256, 0, st>>>(
+        reinterpret_cast<const uint16_t *>(o), reinterpret_cast<const uint16_t *>(dO),
+        const_cast<float *>(p.delta), rows, p.Hq, p.S, p.varlen);
+    if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
+  }
   // dK/dV units: (sequence, key/value head, key tile); dQ units: (sequence,
   // query head, query tile).  Varlen: upper bounds (T + 127 B) / 128 tiles.
   const int64_t tiles = p.varlen ? ((int64_t)p.S + 127LL * p.B) / kTile : (int64_t)p.B * p.n_tiles;
   Params pk = p, pq = p;
   pk.n_units = (int)(tiles * p.Hkv);
   pq.n_units = (int)(tiles * p.Hq);
-  const int gk = pk.n_units < di.sm_count ? pk.n_units : di.sm_count;
-  bwd_kernel<D, false><<<gk, kThreads, Cfg<D>::kSmemBytes, st>>>(tq, tk, tv, tdo, pk);
-  if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
-  const int gq = pq.n_units < di.sm_count ? pq.n_units : di.sm_count;
-  bwd_kernel<D, true><<<gq, kThreads, Cfg<D>::kSmemBytes, st>>>(tq, tk, tv, tdo, pq);
-  return cudaGetLastError() == cudaSuccess ? MK_OK : MK_ERR_CUDA;
+  if (stages & 2) {
+    const int gk = pk.n_units < di.sm_count ? pk.n_units : di.sm_count;
+    bwd_kernel<D, false><<<gk, kThreads, Cfg<D, false>::kSmemBytes, st>>>(tq, tk, tv, tdo, pk);
+    if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
+  }
+  if (stages & 4) {
+    const int gq = pq.n_units < di.sm_count ? pq.n_units : di.sm_count;
+    bwd_kernel<D, true><<<gq, kThreads, Cfg<D, true>::kSmemBytes, st>>>(tq, tk, tv, tdo, pq);
+    if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
+  }
+  return MK_OK;
 }
 
 }  // namespace bwd
@@ -714,11 +803,13 @@ int64_t mk_attn_bwd_workspace_bytes(int B, int Hq, int S, int varlen) {
   return rows * 4;
 }
 
-int mk_attn_bwd(const void *q, const void *k, const void *v, const void *o, const float *lse,
-                const void *dO, void *dq, void *dk, void *dv, int B, int Hq, int Hkv, int S,
-                int D, int causal, float scale, const int32_t *cu_seqlens, void *workspace,
-                int64_t workspace_bytes, void *stream) {
+int mk_attn_bwd_stages(const void *q, const void *k, const void *v, const void *o,
+                       const float *lse, const void *dO, void *dq, void *dk, void *dv, int B,
+                       int Hq, int Hkv, int S, int D, int causal, float scale,
+                       const int32_t *cu_seqlens, void *workspace, int64_t workspace_bytes,
+                       int stages, void *stream) {
   using namespace mk;
+  if (stages < 1 || stages > MK_BWD_ALL) return MK_ERR_INVALID_ARG;
   if (!q || !k || !v || !o || !lse || !dO || !dq || !dk || !dv || !workspace)
     return MK_ERR_INVALID_ARG;
   if (B < 1 || Hq < 1 || Hkv < 1 || S < 1 || Hq % Hkv != 0) return MK_ERR_INVALID_ARG;
@@ -758,8 +849,16 @@ int mk_attn_bwd(const void *q, const void *k, const void *v, const void *o, cons
   p.scale = scale;
   p.scale_log2 = scale * 1.4426950408889634f;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  if (D == 128) return bwd::launch<128>(q, k, v, o, dO, p, tokens, st);
-  return bwd::launch<64>(q, k, v, o, dO, p, tokens, st);
+  if (D == 128) return bwd::launch<128>(q, k, v, o, dO, p, tokens, stages, st);
+  return bwd::launch<64>(q, k, v, o, dO, p, tokens, stages, st);
+}
+
+int mk_attn_bwd(const void *q, const void *k, const void *v, const void *o, const float *lse,
+                const void *dO, void *dq, void *dk, void *dv, int B, int Hq, int Hkv, int S,
+                int D, int causal, float scale, const int32_t *cu_seqlens, void *workspace,
+                int64_t workspace_bytes, void *stream) {
+  return mk_attn_bwd_stages(q, k, v, o, lse, dO, dq, dk, dv, B, Hq, Hkv, S, D, causal, scale,
+                            cu_seqlens, workspace, workspace_bytes, MK_BWD_ALL, stream);
 }
 
 }  // extern "C"
