@@ -134,7 +134,8 @@ MK_API int64_t mk_attn_bwd_workspace_bytes(int B, int Hq, int S, int varlen);
  * Layout and alignment: as mk_attn_fwd; dO, dq, dk, dv and workspace 16-byte
  * aligned, lse 4-byte aligned.
  * Returns MK_OK, or MK_ERR_INVALID_ARG (null pointer, sizes, too small a
- * workspace), MK_ERR_UNSUPPORTED (D), MK_ERR_ALIGNMENT, MK_ERR_CUDA; on any
+ * workspace), MK_ERR_UNSUPPORTED (D, or Hq above 65535), MK_ERR_ALIGNMENT,
+ * MK_ERR_CUDA; on any
  * error nothing is enqueued.  Deterministic: no atomics, repeated calls give
  * bitwise identical gradients.  Internal waits are bounded as in mk_attn_fwd
  * (MK_ERR_TIMEOUT through mk_attn_check_status).

@@ -73,6 +73,17 @@ constexpr float kLog2e = 1.4426950408889634f;
 
 __device__ int g_status = 0;  // MK_ERR_TIMEOUT once a wait ran out
 
+// 32 lanes x 16 columns of 32-bit words from registers into TMEM (the warp's
+// lane quarter), asynchronous until tcgen05.wait::st.
+__device__ __forceinline__ void tmem_st_x16(uint32_t taddr, const uint32_t *r) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
+}
+
 // Ring depths: Y1 is the load on the critical path (its slot frees only when
 // the last MMA of an iteration has read it), so it gets the deeper ring where
 // shared memory allows: at D = 128 the dQ kernel has room for three Y1
@@ -589,11 +600,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int c = 0; c < 64; ++c) x[c] = (row > col0 + c) ? 0.f : x[c];
           }
-          // P^T (bf16) into the first 32 columns of this half of S.
+          // P^T (bf16) into the first 32 columns of this half of S, in two
+          // stores so that the first one's latency overlaps the second pack.
           uint32_t pk[32];
 #pragma unroll
-          for (int c = 0; c < 32; ++c) pk[c] = pack_bf16x2(x[2 * c], x[2 * c + 1]);
-          tmem_st_32x32b_x32(t_row + kColS + col0, pk);
+          for (int c = 0; c < 16; ++c) pk[c] = pack_bf16x2(x[2 * c], x[2 * c + 1]);
+          tmem_st_x16(t_row + kColS + col0, pk);
+#pragma unroll
+          for (int c = 16; c < 32; ++c) pk[c] = pack_bf16x2(x[2 * c], x[2 * c + 1]);
+          tmem_st_x16(t_row + kColS + col0 + 16, pk + 16);
           tmem_st_wait();
           tc_fence_before_sync();
           mbar_arrive(&ctl->p_full);
@@ -613,24 +628,29 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_before_sync();
             mbar_arrive(&ctl->dp_free);
           }
+          // dK/dV: dS^T in place of dP^T; dQ: dS into buffer i % 2.  Two
+          // stores of 32 keys each, the first overlapping the second half.
+          const uint32_t t_ds = t_row + (DQ ? kColAcc + D + (i & 1) * 64 + wg * 32 : kColP + col0);
           uint32_t pk[32];
 #pragma unroll
-          for (int c = 0; c < 64; c += 4) {
-            float4 d4;
-            if constexpr (DQ) {
-              d4 = make_float4(row_dl, row_dl, row_dl, row_dl);
-            } else {
-              d4 = *reinterpret_cast<const float4 *>(lv + kTile + col0 + c);
+          for (int hh = 0; hh < 2; ++hh) {
+#pragma unroll
+            for (int c = hh * 32; c < hh * 32 + 32; c += 4) {
+              float4 d4;
+              if constexpr (DQ) {
+                d4 = make_float4(row_dl, row_dl, row_dl, row_dl);
+              } else {
+                d4 = *reinterpret_cast<const float4 *>(lv + kTile + col0 + c);
+              }
+              const float ds0 = x[c] * (__uint_as_float(raw[c / 32][c % 32]) - d4.x);
+              const float ds1 = x[c + 1] * (__uint_as_float(raw[c / 32][c % 32 + 1]) - d4.y);
+              const float ds2 = x[c + 2] * (__uint_as_float(raw[c / 32][c % 32 + 2]) - d4.z);
+              const float ds3 = x[c + 3] * (__uint_as_float(raw[c / 32][c % 32 + 3]) - d4.w);
+              pk[c / 2] = pack_bf16x2(ds0, ds1);
+              pk[c / 2 + 1] = pack_bf16x2(ds2, ds3);
             }
-            const float ds0 = x[c] * (__uint_as_float(raw[c / 32][c % 32]) - d4.x);
-            const float ds1 = x[c + 1] * (__uint_as_float(raw[c / 32][c % 32 + 1]) - d4.y);
-            const float ds2 = x[c + 2] * (__uint_as_float(raw[c / 32][c % 32 + 2]) - d4.z);
-            const float ds3 = x[c + 3] * (__uint_as_float(raw[c / 32][c % 32 + 3]) - d4.w);
-            pk[c / 2] = pack_bf16x2(ds0, ds1);
-            pk[c / 2 + 1] = pack_bf16x2(ds2, ds3);
+            tmem_st_x16(t_ds + hh * 16, pk + hh * 16);
           }
-          // dK/dV: dS^T in place of dP^T; dQ: dS into buffer i % 2.
-          tmem_st_32x32b_x32(t_row + (DQ ? kColAcc + D + (i & 1) * 64 + wg * 32 : kColP + col0), pk);
           tmem_st_wait();
         }
         tc_fence_before_sync();
@@ -686,18 +706,21 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0 && ctl->abort) atomicExch(&g_status, (int)MK_ERR_TIMEOUT);
 }
 
-// Delta_i = dO_i . o_i in fp32, one half-warp per (token, query head) row,
-// written with the layout of lse.
+// Delta_i = dO_i . o_i in fp32, one half-warp per (token, query head) row:
+// block (x, y) takes tokens 16 x .. 16 x + 15 of query head y, so that the
+// Delta writes of a block are contiguous in the layout of lse.
 template <int D>
 __global__ void __launch_bounds__(256) delta_kernel(const uint16_t *o, const uint16_t *dO,
-                                                    float *delta, int64_t rows, int Hq, int S,
+                                                    float *delta, int tokens, int Hq, int S,
                                                     int varlen) {
-  const int64_t r = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / 16;
+  const int tok = blockIdx.x * 16 + (int)(threadIdx.x >> 4);
+  const int h = blockIdx.y;
   const int l16 = threadIdx.x & 15;
   float acc = 0.f;
-  if (r < rows && l16 * 8 < D) {
-    const uint4 a = *reinterpret_cast<const uint4 *>(o + r * D + l16 * 8);
-    const uint4 b = *reinterpret_cast<const uint4 *>(dO + r * D + l16 * 8);
+  if (tok < tokens && l16 * 8 < D) {
+    const int64_t off = ((int64_t)tok * Hq + h) * D + l16 * 8;
+    const uint4 a = *reinterpret_cast<const uint4 *>(o + off);
+    const uint4 b = *reinterpret_cast<const uint4 *>(dO + off);
     const uint32_t aw[4] = {a.x, a.y, a.z, a.w}, bw[4] = {b.x, b.y, b.z, b.w};
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
@@ -707,10 +730,14 @@ __global__ void __launch_bounds__(256) delta_kernel(const uint16_t *o, const uin
   }
 #pragma unroll
   for (int off = 8; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
-  if (r < rows && l16 == 0) {
-    const int64_t tok = r / Hq;
-    const int h = (int)(r % Hq);
-    const int64_t idx = varlen ? (int64_t)h * S + tok : ((tok / S) * Hq + h) * S + tok % S;
+  if (tok < tokens && l16 == 0) {
+    int64_t idx;
+    if (varlen) {
+      idx = (int64_t)h * S + tok;
+    } else {
+      const int b = tok / S;
+      idx = ((int64_t)b * Hq + h) * S + (tok - b * S);
+    }
     delta[idx] = acc;
   }
 }
@@ -755,11 +782,11 @@ static int launch(const void *q, const void *k, const void *v, const void *o, co
   const int v0 = D == 128 ? 2 : 0;
   if (di.sm_count <= 0 || di.attr_err[v0] != cudaSuccess || di.attr_err[v0 + 1] != cudaSuccess)
     return MK_ERR_CUDA;
-  const int64_t rows = tokens * p.Hq;
   if (stages & 1) {
-    delta_kernel<D><<<(unsigned)((rows * 16 + 255) / 256), 256, 0, st>>>(
+    const dim3 grid((unsigned)((tokens + 15) / 16), (unsigned)p.Hq);
+    delta_kernel<D><<<grid, 256, 0, st>>>(
         reinterpret_cast<const uint16_t *>(o), reinterpret_cast<const uint16_t *>(dO),
-        const_cast<float *>(p.delta), rows, p.Hq, p.S, p.varlen);
+        const_cast<float *>(p.delta), (int)tokens, p.Hq, p.S, p.varlen);
     if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
   }
   // dK/dV units: (sequence, key/value head, key tile); dQ units: (sequence,
@@ -815,6 +842,7 @@ int mk_attn_bwd_stages(const void *q, const void *k, const void *v, const void *
   if (B < 1 || Hq < 1 || Hkv < 1 || S < 1 || Hq % Hkv != 0) return MK_ERR_INVALID_ARG;
   if (!std::isfinite(scale)) return MK_ERR_INVALID_ARG;
   if (D != 64 && D != 128) return MK_ERR_UNSUPPORTED;
+  if (Hq > 65535) return MK_ERR_UNSUPPORTED;  // the Delta kernel's grid y
   const bool varlen = cu_seqlens != nullptr;
   const int64_t tokens = varlen ? (int64_t)S : (int64_t)B * S;
   if (tokens > INT32_MAX || tokens * Hq > INT32_MAX) return MK_ERR_INVALID_ARG;
