@@ -220,9 +220,9 @@ MK_API int mk_attn_decode_paged(const void *q, const void *k_cache, const void *
                                 int max_pages, int num_pages, float scale, void *workspace,
                                 int64_t workspace_bytes, void *stream);
 
-/* Size of the library's own decode scratch array (8 MiB), which every GPU
+/* Size of the library's own decode scratch array (16 MiB), which every GPU
  * that loads the library holds until the process exits. */
-#define MK_ATTN_DECODE_STATIC_SCRATCH_BYTES (8 * 1024 * 1024)
+#define MK_ATTN_DECODE_STATIC_SCRATCH_BYTES (16 * 1024 * 1024)
 
 /*
  * mk_attn_decode_paged_noalloc -- mk_attn_decode_paged for callers that
@@ -255,6 +255,47 @@ MK_API int mk_attn_decode_paged_noalloc(const void *q, const void *k_cache, cons
                                         void *o, float *lse, int B, int Hq, int Hkv, int D,
                                         int page_size, int max_pages, int num_pages, float scale,
                                         void *stream);
+
+/* Schedules of work units over the persistent CTAs (mk_attn_tuning.schedule).
+ * Units are numbered heaviest first (causal: the query tiles that see the most
+ * keys, or the key tiles seen by the most queries). */
+#define MK_SCHED_SNAKE 0       /* round k: CTA c takes unit kG + c, or kG + G-1-c in odd rounds */
+#define MK_SCHED_ROUND_ROBIN 1 /* round k: CTA c takes unit kG + c */
+#define MK_SCHED_BLOCKED 2     /* CTA c takes units c*ceil(n/G) .. (c+1)*ceil(n/G) - 1 */
+
+/*
+ * Launch parameters that change speed but never results beyond rounding:
+ * the knobs of the config autotuner (the paper's Autotuning Agent, Section
+ * 2.1, searches kernel configurations the same way: time each candidate,
+ * keep the fastest correct one).  Tile shapes and pipeline depths are fixed
+ * at compile time by TMEM and shared-memory capacity and are not tunable.
+ */
+typedef struct {
+  int ctas;              /* forward / backward: persistent CTAs, 0 = one per SM;
+                            otherwise 1..65535 (capped at the number of units) */
+  int schedule;          /* forward / backward: MK_SCHED_* */
+  float rescale_log2;    /* forward: the running row max moves (and O is rescaled)
+                            only when it rises by more than this, in log2 units;
+                            0..16, exact for every value (default 8) */
+  int split_ctas_per_sm; /* decode: KV splits are planned for about this many
+                            CTAs per SM, 1..64 (default 24) */
+  int split_min_pages;   /* decode: fewest pages per KV split, 1..4096 (default 2) */
+} mk_attn_tuning;
+
+/*
+ * mk_attn_set_tuning -- sets the process-wide tuning used by every later
+ * call of mk_attn_fwd, mk_attn_bwd(_stages), mk_attn_decode_paged(_noalloc)
+ * and mk_attn_decode_workspace_bytes (the decode split plan, and so its
+ * workspace size, depends on it).  NULL restores the defaults.  Returns
+ * MK_OK, or MK_ERR_INVALID_ARG for a value out of range (the settings are
+ * then unchanged).  Host only; thread-safe, but a call racing a launch on
+ * another thread may apply to it or not.
+ */
+MK_API int mk_attn_set_tuning(const mk_attn_tuning *tuning);
+
+/* mk_attn_get_tuning -- copies the current tuning into *tuning (MK_OK), or
+ * returns MK_ERR_INVALID_ARG for NULL. */
+MK_API int mk_attn_get_tuning(mk_attn_tuning *tuning);
 
 /* Short static description of a status code.  Never NULL. */
 MK_API const char *mk_attn_error_string(int status);

@@ -24,15 +24,33 @@ MK_ERR_SCRATCH_LIMIT = -6
 # Backward-pass stages (MK_BWD_* in include/mk_attn.h).
 BWD_DELTA, BWD_DKDV, BWD_DQ, BWD_ALL = 1, 2, 4, 7
 
+# Unit schedules (MK_SCHED_*).
+SCHED_SNAKE, SCHED_ROUND_ROBIN, SCHED_BLOCKED = 0, 1, 2
+
+
+class MkAttnTuning(ctypes.Structure):
+    """mk_attn_tuning: launch parameters that change speed, not results."""
+    _fields_ = [("ctas", ctypes.c_int), ("schedule", ctypes.c_int),
+                ("rescale_log2", ctypes.c_float), ("split_ctas_per_sm", ctypes.c_int),
+                ("split_min_pages", ctypes.c_int)]
+
+    def as_dict(self) -> dict:
+        return {name: getattr(self, name) for name, _ in self._fields_}
+
+
+DEFAULT_TUNING = dict(ctas=0, schedule=SCHED_SNAKE, rescale_log2=8.0, split_ctas_per_sm=24,
+                      split_min_pages=2)
+
 # Bytes of the library's own decode scratch array (MK_ATTN_DECODE_STATIC_SCRATCH_BYTES).
-DECODE_STATIC_SCRATCH_BYTES = 8 * 1024 * 1024
+DECODE_STATIC_SCRATCH_BYTES = 16 * 1024 * 1024
 
 # Symbols declared in include/mk_attn.h.
 EXPORTED = ("mk_attn_fwd", "mk_attn_fwd_stall_test", "mk_attn_bwd_workspace_bytes", "mk_attn_bwd",
             "mk_attn_bwd_stages",
             "mk_attn_decode_workspace_bytes",
             "mk_attn_decode_paged", "mk_attn_decode_paged_noalloc", "mk_attn_error_string",
-            "mk_attn_check_status", "mk_attn_version")
+            "mk_attn_check_status", "mk_attn_version", "mk_attn_set_tuning",
+            "mk_attn_get_tuning")
 
 _lock = threading.Lock()
 _lib = None
@@ -86,6 +104,10 @@ def load_library() -> ctypes.CDLL:
             lib.mk_attn_check_status.restype = i
             lib.mk_attn_version.argtypes = []
             lib.mk_attn_version.restype = i
+            lib.mk_attn_set_tuning.argtypes = [ctypes.POINTER(MkAttnTuning)]
+            lib.mk_attn_set_tuning.restype = i
+            lib.mk_attn_get_tuning.argtypes = [ctypes.POINTER(MkAttnTuning)]
+            lib.mk_attn_get_tuning.restype = i
             _lib = lib
     return _lib
 
@@ -115,6 +137,44 @@ def mk_attn_check_status(stream: int | None) -> int:
 
 def mk_attn_version() -> int:
     return load_library().mk_attn_version()
+
+
+def mk_attn_set_tuning(tuning: MkAttnTuning | None) -> int:
+    """Raw C-ABI call; None restores the defaults."""
+    return load_library().mk_attn_set_tuning(None if tuning is None else ctypes.byref(tuning))
+
+
+def mk_attn_get_tuning() -> MkAttnTuning:
+    t = MkAttnTuning()
+    _check(load_library().mk_attn_get_tuning(ctypes.byref(t)))
+    return t
+
+
+def set_tuning(**fields) -> None:
+    """Sets the process-wide tuning: the defaults, overridden by `fields`
+    (ctas, schedule, rescale_log2, split_ctas_per_sm, split_min_pages)."""
+    unknown = set(fields) - set(DEFAULT_TUNING)
+    if unknown:
+        raise ValueError(f"unknown tuning fields {sorted(unknown)}")
+    _check(mk_attn_set_tuning(MkAttnTuning(**{**DEFAULT_TUNING, **fields})))
+
+
+class tuning:
+    """Context manager: `with tuning(ctas=120): ...` applies a tuning and
+    restores the previous one on exit."""
+
+    def __init__(self, **fields):
+        self.fields = fields
+        self.saved = None
+
+    def __enter__(self):
+        self.saved = mk_attn_get_tuning()
+        set_tuning(**self.fields)
+        return self
+
+    def __exit__(self, *exc):
+        _check(mk_attn_set_tuning(self.saved))
+        return False
 
 
 def _check(status: int):

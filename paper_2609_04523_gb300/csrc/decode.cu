@@ -53,8 +53,8 @@ namespace dec {
 constexpr int kWarps = 4;                    // compute warps
 constexpr int kThreads = 32 * (kWarps + 1);  // + one producer warp
 constexpr int kMaxStages = 8;
-constexpr int kTargetCtasPerSm = 12;         // split planning: aim for this many CTAs per SM
-constexpr int kMinPagesPerSplit = 4;
+// Split planning (defaults of mk_attn_tuning): aim for about 24 CTAs per SM,
+// and no split shorter than 2 pages.
 
 __device__ int g_status = 0;  // MK_ERR_TIMEOUT or MK_ERR_INVALID_ARG from a decode launch
 
@@ -497,17 +497,19 @@ static void head_split(int G, int &HG, int &head_groups) {
 }
 
 // Splits per (b, g, head group): pages_per_split pages each, so that there
-// are about kTargetCtasPerSm CTAs per SM (several waves of them, so that
+// are about split_ctas_per_sm CTAs per SM (several waves of them, so that
 // sequences of different lengths even out), but no split shorter than
-// kMinPagesPerSplit pages and no more splits than the longest possible
-// sequence has pages.
+// split_min_pages pages and no more splits than the longest possible
+// sequence has pages (both from the process-wide tuning).
 static void plan_splits(int B, int Hkv, int head_groups, int max_pages, int sms, int &n_splits,
                         int &pps) {
+  const mk_attn_tuning tune = current_tuning();
   const int64_t units = (int64_t)B * Hkv * head_groups;
-  int64_t want = (kTargetCtasPerSm * (int64_t)sms + units - 1) / units;
+  int64_t want = ((int64_t)tune.split_ctas_per_sm * sms + units - 1) / units;
   want = want < 1 ? 1 : (want > max_pages ? max_pages : want);
   pps = (int)((max_pages + want - 1) / want);
-  if (pps < kMinPagesPerSplit) pps = kMinPagesPerSplit < max_pages ? kMinPagesPerSplit : max_pages;
+  const int min_pages = tune.split_min_pages;
+  if (pps < min_pages) pps = min_pages < max_pages ? min_pages : max_pages;
   n_splits = (max_pages + pps - 1) / pps;
 }
 

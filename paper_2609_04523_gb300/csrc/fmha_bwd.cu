@@ -128,6 +128,7 @@ struct Params {
   int causal, varlen;
   int n_tiles;               // fixed length: 128-row tiles per sequence
   int n_units;
+  int schedule;              // MK_SCHED_*
   float scale, scale_log2;
 };
 
@@ -214,8 +215,15 @@ __device__ __forceinline__ int unit_iters(const Params &p, const Unit &w, int &f
   }
 }
 
-__device__ __forceinline__ int unit_of_round(int k) {
+// Unit of this CTA in round k (MK_SCHED_*; snake by default, as in the
+// forward kernel); an index >= n_units means no unit.
+__device__ __forceinline__ int unit_of_round(int k, int schedule, int n_units) {
   const int G = gridDim.x, c = blockIdx.x;
+  if (schedule == MK_SCHED_BLOCKED) {
+    const int per = (n_units + G - 1) / G;
+    return k < per ? c * per + k : n_units;
+  }
+  if (schedule == MK_SCHED_ROUND_ROBIN) return k * G + c;
   return (k & 1) ? (k + 1) * G - 1 - c : k * G + c;
 }
 
@@ -296,7 +304,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_load_3d(dst + hb * kBoxBytes, map, bar, hb * kBoxCols, head, row0, pol);
     };
     for (int k = 0; ok && k * (int)gridDim.x < p.n_units; ++k) {
-      const int u = unit_of_round(k);
+      const int u = unit_of_round(k, p.schedule, p.n_units);
       if (u >= p.n_units) continue;
       const Unit w = map_unit<DQ>(p, u);
       if (!w.valid) continue;
@@ -422,7 +430,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     };
     for (int k = 0; ok && k * (int)gridDim.x < p.n_units; ++k) {
-      const int u = unit_of_round(k);
+      const int u = unit_of_round(k, p.schedule, p.n_units);
       if (u >= p.n_units) continue;
       const Unit w = map_unit<DQ>(p, u);
       if (!w.valid) continue;
@@ -533,7 +541,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     constexpr uint32_t kColAcc2 = DQ ? kColAcc : kColAcc + D;
     static_assert(!DQ || kColAcc + D + 128 <= kTmemCols, "dS buffers");
     for (int k = 0; ok && k * (int)gridDim.x < p.n_units; ++k) {
-      const int u = unit_of_round(k);
+      const int u = unit_of_round(k, p.schedule, p.n_units);
       if (u >= p.n_units) continue;
       const Unit w = map_unit<DQ>(p, u);
       if (!w.valid) continue;
@@ -792,16 +800,19 @@ static int launch(const void *q, const void *k, const void *v, const void *o, co
   // dK/dV units: (sequence, key/value head, key tile); dQ units: (sequence,
   // query head, query tile).  Varlen: upper bounds (T + 127 B) / 128 tiles.
   const int64_t tiles = p.varlen ? ((int64_t)p.S + 127LL * p.B) / kTile : (int64_t)p.B * p.n_tiles;
+  const mk_attn_tuning tune = current_tuning();
+  const int ctas = tune.ctas > 0 ? tune.ctas : di.sm_count;
+  p.schedule = tune.schedule;
   Params pk = p, pq = p;
   pk.n_units = (int)(tiles * p.Hkv);
   pq.n_units = (int)(tiles * p.Hq);
   if (stages & 2) {
-    const int gk = pk.n_units < di.sm_count ? pk.n_units : di.sm_count;
+    const int gk = pk.n_units < ctas ? pk.n_units : ctas;
     bwd_kernel<D, false><<<gk, kThreads, Cfg<D, false>::kSmemBytes, st>>>(tq, tk, tv, tdo, pk);
     if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
   }
   if (stages & 4) {
-    const int gq = pq.n_units < di.sm_count ? pq.n_units : di.sm_count;
+    const int gq = pq.n_units < ctas ? pq.n_units : ctas;
     bwd_kernel<D, true><<<gq, kThreads, Cfg<D, true>::kSmemBytes, st>>>(tq, tk, tv, tdo, pq);
     if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
   }

@@ -35,7 +35,8 @@
 // MMA warp issues P_X V over keys 0..63 while keys 64..127 are exponentiated.
 // Because S_X(j) is issued after P_X(j-1) V_{j-1}, every MMA that touches O_X
 // has completed when S_X(j) has: the softmax warps rescale O_X in TMEM (lazily,
-// only when the row max rises by more than kRescaleThreshold) with no extra wait.
+// only when the row max rises by more than a threshold, 8 in log2 units by
+// default) with no extra wait.
 // Softmax: base-2 online softmax in fp32 (t = s * scale * log2 e, ex2 on the
 // MUFU unit), P rounded to bf16 (RNE); epilogue o = O / l -> bf16,
 // lse = ln 2 * (m + log2 l).  Causal tiles visit key blocks 0..qt only and mask
@@ -70,7 +71,6 @@ constexpr int kBoxBytes = kTile * kBoxCols * 2;  // one TMA box: 128 rows x 128 
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColS = 0;         // S_X at kColS + 128 * X
 constexpr uint32_t kColO = 256;       // O_X at kColO + D * X
-constexpr float kRescaleThreshold = 8.0f;  // log2 units: rescale O when m rises by > 2^8
 constexpr int kCuCache = 2048;        // cu_seqlens entries cached in shared memory
 constexpr int kMaxLevels = 1024;      // causal varlen: longest-first order up to 1024 tile pairs
                                       // (262144 tokens) per sequence
@@ -133,6 +133,8 @@ struct Params {
   float scale_log2;         // scale * log2(e)
   int o_align32;            // o is 32-byte aligned: 256-bit stores in the epilogue
   int stall_first_slot;     // failure-path test: the producer loads nothing
+  int schedule;             // MK_SCHED_*: units over the persistent CTAs
+  float rescale_log2;       // lazy O rescale threshold (log2 units)
 };
 
 __device__ __forceinline__ int clamp_tok(int x, int T) { return x < 0 ? 0 : (x > T ? T : x); }
@@ -287,11 +289,18 @@ __device__ __forceinline__ int tile_blocks(const Params &p, const Unit &w, int X
 }
 
 // Unit processed by this CTA in round k.  Units are numbered heaviest first
-// (fixed-length causal); rounds alternate direction over the CTAs (CTA c takes
-// unit kG + c in even rounds and kG + G - 1 - c in odd ones), which balances
-// the per-CTA sums of decreasing unit costs far better than plain round-robin.
-__device__ __forceinline__ int unit_of_round(int k) {
+// (fixed-length causal).  The default (snake) alternates the direction of the
+// rounds over the CTAs (CTA c takes unit kG + c in even rounds and
+// kG + G - 1 - c in odd ones), which balances the per-CTA sums of decreasing
+// unit costs far better than plain round-robin; blocked gives each CTA a
+// contiguous run of units.  A unit index >= n_units means no unit.
+__device__ __forceinline__ int unit_of_round(int k, int schedule, int n_units) {
   const int G = gridDim.x, c = blockIdx.x;
+  if (schedule == MK_SCHED_BLOCKED) {
+    const int per = (n_units + G - 1) / G;
+    return k < per ? c * per + k : n_units;
+  }
+  if (schedule == MK_SCHED_ROUND_ROBIN) return k * G + c;
   return (k & 1) ? (k + 1) * G - 1 - c : k * G + c;
 }
 
@@ -414,7 +423,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       bool ok = true;
       for (int k = 0; ok && k * (int)gridDim.x < p.n_units; ++k) {
-        const int u = unit_of_round(k);
+        const int u = unit_of_round(k, p.schedule, p.n_units);
         if (u >= p.n_units) continue;
         const Unit w = map_unit<VL>(p, cu_smem, sched, u);
         if (!w.valid) continue;
@@ -698,7 +707,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // Lazy rescaling: keep the old reference max unless the new one exceeds
         // it by more than the threshold.  Exact either way, because O and l
         // always share the same reference max.
-        const bool rescale = m_new > m_run + kRescaleThreshold;
+        const bool rescale = m_new > m_run + p.rescale_log2;
         float alpha = 1.f;
         if (rescale) {
           alpha = ex2_approx(m_run - m_new);  // 0 when m_run = -inf
@@ -861,7 +870,9 @@ static int launch(const void *q, const void *k, const void *v, const Params &p, 
   // kLaunchRegs registers per thread; anything else could leave a
   // setmaxnreg.inc waiting forever, so refuse to launch.
   if (di.regs[vi] != kLaunchRegs) return MK_ERR_CUDA;
-  const int grid = p.n_units < di.sm_count ? p.n_units : di.sm_count;
+  const mk_attn_tuning tune = current_tuning();
+  const int ctas = tune.ctas > 0 ? tune.ctas : di.sm_count;
+  const int grid = p.n_units < ctas ? p.n_units : ctas;
   fmha_fwd_kernel<D, VL><<<grid, kThreads, C::kSmemBytes, stream>>>(tq, tk, tv, p);
   return cudaGetLastError() == cudaSuccess ? MK_OK : MK_ERR_CUDA;
 }
@@ -919,6 +930,9 @@ static int attn_fwd_impl(const void *q, const void *k, const void *v, void *o, f
   p.scale_log2 = scale * 1.4426950408889634f;
   p.o_align32 = (reinterpret_cast<uintptr_t>(o) & 31u) == 0;
   p.stall_first_slot = stall_first_slot;
+  const mk_attn_tuning tune = current_tuning();
+  p.schedule = tune.schedule;
+  p.rescale_log2 = tune.rescale_log2;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (D == 128)
     return varlen ? launch<128, true>(q, k, v, p, tokens, st) : launch<128, false>(q, k, v, p, tokens, st);

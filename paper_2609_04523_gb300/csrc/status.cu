@@ -2,8 +2,23 @@
 // the device status check that covers every kernel family, and the version.
 #include <cuda_runtime.h>
 
+#include <mutex>
+
 #include "mk_attn.h"
 #include "tma_host.h"
+
+namespace mk {
+namespace {
+constexpr mk_attn_tuning kDefaultTuning = {0, MK_SCHED_SNAKE, 8.0f, 24, 2};
+std::mutex g_tuning_mu;
+mk_attn_tuning g_tuning = kDefaultTuning;
+}  // namespace
+
+mk_attn_tuning current_tuning() {
+  std::lock_guard<std::mutex> lock(g_tuning_mu);
+  return g_tuning;
+}
+}  // namespace mk
 
 extern "C" {
 
@@ -31,6 +46,27 @@ int mk_attn_check_status(void *stream) {
   return hf != 0 ? hf : (hb != 0 ? hb : hd);
 }
 
-int mk_attn_version(void) { return 400; }
+int mk_attn_set_tuning(const mk_attn_tuning *t) {
+  mk_attn_tuning v = mk::kDefaultTuning;
+  if (t) {
+    if (t->ctas < 0 || t->ctas > 65535) return MK_ERR_INVALID_ARG;
+    if (t->schedule < MK_SCHED_SNAKE || t->schedule > MK_SCHED_BLOCKED) return MK_ERR_INVALID_ARG;
+    if (!(t->rescale_log2 >= 0.0f && t->rescale_log2 <= 16.0f)) return MK_ERR_INVALID_ARG;
+    if (t->split_ctas_per_sm < 1 || t->split_ctas_per_sm > 64) return MK_ERR_INVALID_ARG;
+    if (t->split_min_pages < 1 || t->split_min_pages > 4096) return MK_ERR_INVALID_ARG;
+    v = *t;
+  }
+  std::lock_guard<std::mutex> lock(mk::g_tuning_mu);
+  mk::g_tuning = v;
+  return MK_OK;
+}
+
+int mk_attn_get_tuning(mk_attn_tuning *t) {
+  if (!t) return MK_ERR_INVALID_ARG;
+  *t = mk::current_tuning();
+  return MK_OK;
+}
+
+int mk_attn_version(void) { return 500; }
 
 }  // extern "C"

@@ -8,6 +8,8 @@
 #include <cstdint>
 #include <mutex>
 
+#include "mk_attn.h"
+
 namespace mk {
 
 // cuTensorMapEncodeTiled through the runtime's driver entry point (no -lcuda).
@@ -39,6 +41,9 @@ inline bool encode_tokens_heads_dim(CUtensorMap *map, const void *base, uint64_t
              box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
+
+// The process-wide launch tuning (mk_attn_set_tuning), defaults applied.
+mk_attn_tuning current_tuning();
 
 // Read and clear the device status word of each kernel family (each defined
 // with its kernels).

@@ -3,7 +3,7 @@
 mk_attn_decode_paged_noalloc serves callers that cannot allocate device
 memory (code running under an allocator that another runtime owns, inside
 host callbacks, or in plugins that must not grow the device heap): its split
-partials go to a fixed 8 MiB array that the library declares in device
+partials go to a fixed 16 MiB array that the library declares in device
 memory instead of a caller workspace.  These tests call it through the C ABI
 and check it against mk_attn_decode_paged with a workspace, within the decode
 tests' tolerances, on two calls in a row (the second sees what the first left
