@@ -77,6 +77,9 @@ def _bind(lib: ctypes.CDLL) -> ctypes.CDLL:
                                                       ctypes.c_double, p, p, ctypes.c_int64, p,
                                                       p, i]
     lib.mk_oracle_attn_bwd_dkv_ranges_f64.restype = i
+    lib.mk_oracle_mla_decode_f64.argtypes = [p, p, p, p, p, p, i, i, i, i, i, i, i,
+                                             ctypes.c_double, i]
+    lib.mk_oracle_mla_decode_f64.restype = i
     return lib
 
 
@@ -261,3 +264,27 @@ def attn_bwd_dkv_ranges(q, k, v, do, causal: bool, scale: float, ranges, cu_seql
     if st != 0:
         raise ValueError(f"oracle rejected the ranges (status {st})")
     return dk, dv
+
+
+def mla_decode(q, cache, page_table, seq_lens, scale: float, dv: int,
+               n_threads: int | None = None, lib: ctypes.CDLL | None = None):
+    """One latent (MLA) decode step in fp64: q [B,Hq,Dqk], cache
+    [num_pages, page_size, Dqk] (keys in full, values = the first dv
+    components), page_table int32 [B, max_pages], seq_lens int32 [B].
+    Returns (o [B,Hq,dv], lse [B,Hq]) as fp64 numpy arrays."""
+    qb, cb = _bits(q), _bits(cache)
+    pt = np.ascontiguousarray(np.asarray(page_table, dtype=np.int32))
+    sl = np.ascontiguousarray(np.asarray(seq_lens, dtype=np.int32))
+    B, Hq, Dqk = qb.shape
+    num_pages, page_size, Dc = cb.shape
+    if Dc != Dqk:
+        raise ValueError("cache rows must have the query's dimension")
+    o = np.zeros((B, Hq, dv), dtype=np.float64)
+    lse = np.zeros((B, Hq), dtype=np.float64)
+    lib = lib or load()
+    st = lib.mk_oracle_mla_decode_f64(_ptr(qb), _ptr(cb), _ptr(pt), _ptr(sl), _ptr(o), _ptr(lse),
+                                      B, Hq, Dqk, dv, page_size, pt.shape[1], num_pages,
+                                      float(scale), int(n_threads or default_threads()))
+    if st != 0:
+        raise ValueError(f"oracle rejected the MLA decode problem (status {st})")
+    return o, lse

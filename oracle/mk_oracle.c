@@ -1,6 +1,7 @@
 /*
  * mk_oracle.c -- plain fp64 CPU oracle for the attention forward pass, its
- * backward pass (gradients of q, k, v) and one paged decode step.
+ * backward pass (gradients of q, k, v), one paged decode step and one latent
+ * (MLA) decode step.
  *
  * TEST INFRASTRUCTURE.  Only tests/, __graft_entry__.smoke() and bench.py's
  * cpu_baseline / reference legs may load this file's library.  The product
@@ -756,4 +757,115 @@ int mk_oracle_attn_bwd_dkv_ranges_f64(const uint16_t *q, const uint16_t *k, cons
     st = run_threads(dkv_range_worker, &job, sizeof job, n_threads);
     free(off);
     return st;
+}
+
+/* ------------------------------------------------- latent (MLA) decode step */
+
+/*
+ * One decode step of multi-head latent attention in its absorbed form: every
+ * query head attends to one shared latent cache (a single key/value head),
+ * whose rows serve as keys in full and as values through their first Dv
+ * components (the paper's MLA Attention row, Table 2 and Table 3).  For
+ * sequence b and query head h, with c_j the cached latent row of position j
+ * (slot j % page_size of page page_table[b, j / page_size]):
+ *
+ *   s_j  = scale * sum_{d < Dqk} q[b,h,d] * c_j[d]
+ *   o[d] = sum_j exp(s_j - m) c_j[d] / sum_j exp(s_j - m),  d < Dv,  m = max_j s_j
+ *   lse  = m + ln(sum_j exp(s_j - m))
+ *
+ * Layouts: q [B, Hq, Dqk]; cache [num_pages, page_size, Dqk]; o [B, Hq, Dv];
+ * lse [B, Hq]; page_table int32 [B, max_pages]; seq_lens int32 [B].
+ * L_b = 0 gives o = 0 and lse = -inf.  Returns MK_ORACLE_BAD_ARG for sizes out
+ * of range (Dv > Dqk included), a length above max_pages * page_size, or a
+ * page index outside [0, num_pages).
+ */
+typedef struct {
+    const uint16_t *q, *cache;
+    const int32_t *page_table, *seq_lens;
+    double *o, *lse;
+    int B, Hq, Dqk, Dv, page_size, max_pages;
+    double scale;
+    int64_t *next;
+    int max_len;
+} mla_job_t;
+
+static const uint16_t *mla_row(const mla_job_t *job, int b, int j)
+{
+    const int64_t page = job->page_table[(int64_t)b * job->max_pages + j / job->page_size];
+    return job->cache + (page * job->page_size + j % job->page_size) * (int64_t)job->Dqk;
+}
+
+static void *mla_worker(void *arg)
+{
+    mla_job_t *job = (mla_job_t *)arg;
+    double *s_buf = (double *)malloc(sizeof(double) * (size_t)(job->max_len > 0 ? job->max_len : 1));
+    if (!s_buf)
+        return NULL;
+    for (;;) {
+        int64_t t = __atomic_fetch_add(job->next, 1, __ATOMIC_RELAXED);
+        if (t >= (int64_t)job->B * job->Hq)
+            break;
+        const int b = (int)(t / job->Hq);
+        const int L = job->seq_lens[b];
+        const uint16_t *qr = job->q + t * (int64_t)job->Dqk;
+        double *orow = job->o + t * (int64_t)job->Dv;
+        for (int d = 0; d < job->Dv; ++d)
+            orow[d] = 0.0;
+        if (L == 0) {
+            job->lse[t] = -INFINITY;
+            continue;
+        }
+        double m = -INFINITY;
+        for (int j = 0; j < L; ++j) {
+            const uint16_t *cj = mla_row(job, b, j);
+            double acc = 0.0;
+            for (int d = 0; d < job->Dqk; ++d)
+                acc += bf16_bits_to_f64(qr[d]) * bf16_bits_to_f64(cj[d]);
+            s_buf[j] = job->scale * acc;
+            if (s_buf[j] > m)
+                m = s_buf[j];
+        }
+        double l = 0.0;
+        for (int j = 0; j < L; ++j) {
+            const double e = exp(s_buf[j] - m);
+            const uint16_t *cj = mla_row(job, b, j);
+            l += e;
+            for (int d = 0; d < job->Dv; ++d)
+                orow[d] += e * bf16_bits_to_f64(cj[d]);
+        }
+        for (int d = 0; d < job->Dv; ++d)
+            orow[d] /= l;
+        job->lse[t] = m + log(l);
+    }
+    free(s_buf);
+    return NULL;
+}
+
+int mk_oracle_mla_decode_f64(const uint16_t *q, const uint16_t *cache, const int32_t *page_table,
+                             const int32_t *seq_lens, double *o, double *lse, int B, int Hq,
+                             int Dqk, int Dv, int page_size, int max_pages, int num_pages,
+                             double scale, int n_threads)
+{
+    if (!q || !cache || !page_table || !seq_lens || !o || !lse)
+        return MK_ORACLE_BAD_ARG;
+    if (B < 1 || Hq < 1 || Dqk < 1 || Dv < 1 || Dv > Dqk || page_size < 1 || max_pages < 1 ||
+        num_pages < 1)
+        return MK_ORACLE_BAD_ARG;
+    int max_len = 0;
+    for (int b = 0; b < B; ++b) {
+        const int L = seq_lens[b];
+        if (L < 0 || (int64_t)L > (int64_t)max_pages * page_size)
+            return MK_ORACLE_BAD_ARG;
+        for (int j = 0; j * page_size < L; ++j) {
+            const int32_t pg = page_table[(int64_t)b * max_pages + j];
+            if (pg < 0 || pg >= num_pages)
+                return MK_ORACLE_BAD_ARG;
+        }
+        if (L > max_len)
+            max_len = L;
+    }
+    int64_t next = 0;
+    mla_job_t job = {q, cache, page_table, seq_lens, o, lse, B, Hq, Dqk, Dv, page_size, max_pages,
+                     scale, &next, max_len};
+    return run_threads(mla_worker, &job, sizeof job, n_threads);
 }

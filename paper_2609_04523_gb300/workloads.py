@@ -291,6 +291,52 @@ def make_paged(seq_lens, Hq: int, Hkv: int, D: int, page_size: int, seed: int,
     return PagedInputs(q, kc, vc, pt, torch.tensor(lens, dtype=torch.int32), 1.0 / math.sqrt(D))
 
 
+@dataclass
+class MlaInputs:
+    q: torch.Tensor           # bf16 [B, Hq, dqk]
+    cache: torch.Tensor       # bf16 [num_pages, page_size, dqk]: latent (dv) + rope (dqk - dv)
+    page_table: torch.Tensor  # int32 [B, max_pages], unused entries -1
+    seq_lens: torch.Tensor    # int32 [B]
+    scale: float
+    dv: int
+
+
+def make_mla_paged(seq_lens, Hq: int, page_size: int, seed: int, dqk: int = 576, dv: int = 512,
+                   sigma: float = 1.0, spare_pages: int = 3,
+                   max_pages: int | None = None) -> MlaInputs:
+    """Seeded inputs of a latent (MLA) decode step: one shared latent cache,
+    pages handed out in a random order as in make_paged.  The scale is
+    1/sqrt(dqk).  Pure data generation: no attention arithmetic."""
+    g = torch.Generator("cpu").manual_seed(seed)
+    lens = [int(x) for x in seq_lens]
+    need = [(L + page_size - 1) // page_size for L in lens]
+    mp = max(1, max(need) if max_pages is None else max_pages)
+    num_pages = sum(need) + spare_pages
+    perm = torch.randperm(num_pages, generator=g).tolist()
+    pt = torch.full((len(lens), mp), -1, dtype=torch.int32)
+    at = 0
+    for b, n in enumerate(need):
+        for j in range(n):
+            pt[b, j] = perm[at]
+            at += 1
+    q = randn_bf16((len(lens), Hq, dqk), g, sigma)
+    cache = randn_bf16((num_pages, page_size, dqk), g, sigma)
+    return MlaInputs(q, cache, pt, torch.tensor(lens, dtype=torch.int32), 1.0 / math.sqrt(dqk), dv)
+
+
+def mla_decode_bytes(seq_lens, Hq: int, dqk: int = 576, dv: int = 512) -> int:
+    """Minimal HBM traffic of one latent decode step: every cached latent row
+    read once (bf16), q read, o written (bf16), lse written."""
+    keys = int(sum(int(x) for x in seq_lens))
+    B = len(seq_lens)
+    return 2 * keys * dqk + 2 * B * Hq * dqk + 2 * B * Hq * dv + 4 * B * Hq
+
+
+def mla_decode_flops(seq_lens, Hq: int, dqk: int = 576, dv: int = 512) -> float:
+    """Matmul FLOPs of one latent decode step: 2 (dqk + dv) per head and key."""
+    return 2.0 * (dqk + dv) * Hq * float(sum(int(x) for x in seq_lens))
+
+
 def decode_bytes(seq_lens, Hq: int, Hkv: int, D: int) -> int:
     """Minimal HBM traffic of one decode step: every cached key and value of
     every sequence read once, q read and o written once (bf16), lse written."""

@@ -609,6 +609,83 @@ def check_bwd_sampled_match_full(lib):
             at += j1 - j0
 
 
+# ------------------------------------------------- latent (MLA) decode step
+
+def _mla(lib, inp):
+    return oracle.mla_decode(inp.q, inp.cache, inp.page_table, inp.seq_lens, inp.scale, inp.dv,
+                             n_threads=2, lib=lib)
+
+
+def _mla_rows(inp, b):
+    """The cached latent rows of sequence b, in position order, fp64."""
+    L = int(inp.seq_lens[b])
+    ps = inp.cache.shape[1]
+    c = _f64(inp.cache)
+    return np.stack([c[int(inp.page_table[b, j // ps]), j % ps] for j in range(L)]) if L else \
+        np.zeros((0, c.shape[2]))
+
+
+def check_mla_library_sdpa(lib):
+    """Library special case: torch's fp64 scaled_dot_product_attention with
+    K = the gathered latent rows and V = their first dv components (SDPA
+    allows a value dimension other than the key's), one key/value head
+    broadcast over the query heads; scipy's logsumexp for the LSE."""
+    from scipy.special import logsumexp
+    for dqk, dv, ps, lens in ((40, 32, 4, [9, 1, 13]), (576, 512, 64, [70, 3])):
+        inp = W.make_mla_paged(lens, 5, ps, seed=161 + dqk, dqk=dqk, dv=dv)
+        o, lse = _mla(lib, inp)
+        for b, L in enumerate(lens):
+            c = torch.from_numpy(_mla_rows(inp, b))
+            q = torch.from_numpy(_f64(inp.q[b]))[None, :, None, :]     # [1, Hq, 1, dqk]
+            k = c[None, None].expand(1, q.shape[1], L, dqk)
+            v = c[None, None, :, :dv].expand(1, q.shape[1], L, dv)
+            ref = torch.nn.functional.scaled_dot_product_attention(q, k, v, scale=inp.scale)
+            _close(o[b], ref[0, :, 0].numpy(), 1e-12, f"mla sdpa o dqk={dqk}")
+            logits = inp.scale * (q[0, :, 0] @ c.T).numpy()
+            _close(lse[b], logsumexp(logits, axis=1), 1e-12, f"mla lse dqk={dqk}")
+
+
+def check_mla_brute_force(lib):
+    """The explicit probability matrix over the gathered rows: o = P V."""
+    inp = W.make_mla_paged([6, 11], 3, 4, seed=171, dqk=24, dv=16)
+    o, lse = _mla(lib, inp)
+    for b in range(2):
+        c = _mla_rows(inp, b)
+        P = brute.probability_matrix(_f64(inp.q[b]), c, False, inp.scale)
+        _close(o[b], P @ c[:, :16], TIGHT, "mla brute o")
+
+
+def check_mla_closed_forms(lib):
+    """One key: o = its first dv components, lse = scale q.c.  Scale 0: o is
+    the mean of the rows' first dv components, lse = ln L.  No key: o = 0,
+    lse = -inf.  Rows permuted across pages: same result."""
+    inp = W.make_mla_paged([1, 0, 37], 4, 8, seed=181, dqk=48, dv=32)
+    o, lse = _mla(lib, inp)
+    c0 = _mla_rows(inp, 0)
+    _close(o[0], np.repeat(c0[:, :32], 4, axis=0), 0.0, "mla single key o")
+    _close(lse[0], inp.scale * (_f64(inp.q[0]) @ c0[0]), 1e-13, "mla single key lse")
+    assert np.all(o[1] == 0.0) and np.all(np.isneginf(lse[1])), "mla empty sequence"
+    z = W.MlaInputs(inp.q, inp.cache, inp.page_table, inp.seq_lens, 0.0, inp.dv)
+    oz, lz = _mla(lib, z)
+    c2 = _mla_rows(inp, 2)
+    _close(oz[2], np.repeat(c2[:, :32].mean(axis=0, keepdims=True), 4, axis=0), 1e-13, "mla scale 0 o")
+    _close(lz[2], np.full(4, math.log(37)), 1e-13, "mla scale 0 lse")
+    # move sequence 2's pages to other physical pages (copying the rows)
+    ps, n = 8, (37 + 7) // 8
+    cache = inp.cache.clone()
+    pt = inp.page_table.clone()
+    free = [p for p in range(cache.shape[0]) if p not in set(int(x) for x in pt[pt >= 0])]
+    moved = list(reversed([int(pt[2, j]) for j in range(n)]))
+    for j in range(n):
+        dst = moved[j]
+        cache[dst] = inp.cache[int(pt[2, j])]
+        pt[2, j] = dst
+    o2, lse2 = _mla(lib, W.MlaInputs(inp.q, cache, pt, inp.seq_lens, inp.scale, inp.dv))
+    _close(o2[2], o[2], TIGHT, "mla page permutation o")
+    _close(lse2[2], lse[2], TIGHT, "mla page permutation lse")
+    del free
+
+
 ALL_CHECKS = [
     check_brute_force_tiny,
     check_brute_force_varlen,
@@ -639,4 +716,7 @@ ALL_CHECKS = [
     check_bwd_gqa_equals_repeated_mha,
     check_bwd_varlen_equals_separate,
     check_bwd_sampled_match_full,
+    check_mla_library_sdpa,
+    check_mla_brute_force,
+    check_mla_closed_forms,
 ]

@@ -40,8 +40,12 @@ MUTANTS = {
         "const int64_t row = (page * job->page_size + j % job->page_size) * job->Hkv + g;\n            const uint16_t *kr",
         "const int64_t row = (page * job->page_size + j / job->page_size) * job->Hkv + g;\n            const uint16_t *kr"),
     "decode_interleaved_groups": ("h = (int)(t % job->Hq), g = h / G;", "h = (int)(t % job->Hq), g = h % job->Hkv;"),
-    "decode_drop_scale": ("s_buf[j] = job->scale * acc;", "s_buf[j] = acc;"),
-    "decode_lse_log2": ("job->lse[t] = m + log(l);", "job->lse[t] = m + log2(l);"),
+    "decode_drop_scale": ("s_buf[j] = job->scale * acc;\n            if (s_buf[j] > m)\n                m = s_buf[j];\n        }\n        double l = 0.0;\n        for (int j = 0; j < L; ++j) {\n            const double e = exp(s_buf[j] - m);\n            l += e;",
+                          "s_buf[j] = acc;\n            if (s_buf[j] > m)\n                m = s_buf[j];\n        }\n        double l = 0.0;\n        for (int j = 0; j < L; ++j) {\n            const double e = exp(s_buf[j] - m);\n            l += e;"),
+    "decode_lse_log2": ("            orow[d] /= l;\n        job->lse[t] = m + log(l);\n    }\n    free(s_buf);\n    return NULL;\n}\n\nint mk_oracle_decode_paged_f64",
+                        "            orow[d] /= l;\n        job->lse[t] = m + log2(l);\n    }\n    free(s_buf);\n    return NULL;\n}\n\nint mk_oracle_decode_paged_f64"),
+    "mla_lse_log2": ("            orow[d] /= l;\n        job->lse[t] = m + log(l);\n    }\n    free(s_buf);\n    return NULL;\n}\n\nint mk_oracle_mla_decode_f64",
+                     "            orow[d] /= l;\n        job->lse[t] = m + log2(l);\n    }\n    free(s_buf);\n    return NULL;\n}\n\nint mk_oracle_mla_decode_f64"),
     "bwd_drop_delta": ("const double dS = P * (dp_buf[j] - delta);\n                    const uint16_t *kj",
                        "const double dS = P * dp_buf[j];\n                    const uint16_t *kj"),
     "bwd_delta_sign": ("delta += s_buf[j] * dp;", "delta -= s_buf[j] * dp;"),
@@ -62,6 +66,14 @@ MUTANTS = {
                                      "return p->causal ? (i < L ? i : L) : L; /* |K_i| */"),
     "bwd_dq_rows_drop_scale": ("dqi[d] += p->scale * dS * bf16_bits_to_f64(kj[d]);\n        }\n    }",
                                "dqi[d] += dS * bf16_bits_to_f64(kj[d]);\n        }\n    }"),
+    "mla_values_from_suffix": ("orow[d] += e * bf16_bits_to_f64(cj[d]);",
+                               "orow[d] += e * bf16_bits_to_f64(cj[d + (job->Dqk - job->Dv)]);"),
+    "mla_rope_dropped": ("for (int d = 0; d < job->Dqk; ++d)\n                acc += bf16_bits_to_f64(qr[d]) * bf16_bits_to_f64(cj[d]);",
+                         "for (int d = 0; d < job->Dv; ++d)\n                acc += bf16_bits_to_f64(qr[d]) * bf16_bits_to_f64(cj[d]);"),
+    "mla_drop_scale": ("s_buf[j] = job->scale * acc;\n            if (s_buf[j] > m)\n                m = s_buf[j];\n        }\n        double l = 0.0;\n        for (int j = 0; j < L; ++j) {\n            const double e = exp(s_buf[j] - m);\n            const uint16_t *cj = mla_row",
+                       "s_buf[j] = acc;\n            if (s_buf[j] > m)\n                m = s_buf[j];\n        }\n        double l = 0.0;\n        for (int j = 0; j < L; ++j) {\n            const double e = exp(s_buf[j] - m);\n            const uint16_t *cj = mla_row"),
+    "mla_slot_from_page_index": ("return job->cache + (page * job->page_size + j % job->page_size) * (int64_t)job->Dqk;",
+                                 "return job->cache + (page * job->page_size + j / job->page_size) * (int64_t)job->Dqk;"),
     "bwd_ranges_skip_first_row": ("for (int i = p->causal ? j0 : 0; i < L; ++i) {",
                                   "for (int i = p->causal ? j0 + 1 : 0; i < L; ++i) {"),
 }
