@@ -22,9 +22,15 @@ dQ kernels) on the same configs, in TFLOP/s of 2.5x the forward's FLOPs (the
 usual convention: five matmuls against the forward's two), and reports the
 dK/dV kernel, timed alone, against the bf16 tensor roofline.
 
+--workload mla times one latent (MLA) decode step (mk_attn_mla_decode_paged:
+64 sequences of 1024-8192 cached tokens, 128 query heads sharing one
+576-wide latent cache, values its first 512 components, page_size=64) in HBM
+GB/s of algorithmic bytes, with its matmul TFLOP/s beside it.
+
 --impl reference times the fp64 CPU oracle on bounded row samples of the same
-workload (the whole step for decode, one sequence for the backward pass;
-rank 0 only; other ranks exit without work).
+workload (the whole step for decode, one sequence for the backward pass,
+leading sequences for the latent decode step; rank 0 only; other ranks exit
+without work).
 """
 from __future__ import annotations
 
@@ -44,11 +50,14 @@ sys.path.insert(0, ROOT)
 METRIC = "attention fwd TFLOP/s (causal FLOPs) and % of GB300 bf16 tensor peak"
 DECODE_METRIC = "paged decode step HBM GB/s (algorithmic bytes) and % of measured HBM copy bandwidth"
 BWD_METRIC = "attention bwd TFLOP/s (2.5x causal forward FLOPs) and % of GB300 bf16 tensor peak"
+MLA_METRIC = ("latent (MLA) decode step HBM GB/s (algorithmic bytes) and % of measured HBM copy "
+              "bandwidth")
 NOMINAL_BF16_TFLOPS = 2250.0
 FLUSH_BYTES = 256 << 20
 KERNEL_SOURCES = ["paper_2609_04523_gb300/csrc/fmha_fwd.cu", "paper_2609_04523_gb300/csrc/ptx.cuh"]
 DECODE_SOURCES = ["paper_2609_04523_gb300/csrc/decode.cu", "paper_2609_04523_gb300/csrc/ptx.cuh"]
 BWD_SOURCES = ["paper_2609_04523_gb300/csrc/fmha_bwd.cu", "paper_2609_04523_gb300/csrc/ptx.cuh"]
+MLA_SOURCES = ["paper_2609_04523_gb300/csrc/mla_decode.cu", "paper_2609_04523_gb300/csrc/ptx.cuh"]
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "ncu_traffic.json")
 BAD_REASONS = {"hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown"}
 
@@ -59,7 +68,8 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5])
-    ap.add_argument("--workload", default="prefill", choices=["prefill", "decode", "backward"],
+    ap.add_argument("--workload", default="prefill",
+                    choices=["prefill", "decode", "backward", "mla"],
                     help="prefill: the attention forward pass (--config); decode: one paged "
                          "decode step (the decode workload below)")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
@@ -919,6 +929,231 @@ def run_backward_reference(args, rank: int):
     }
 
 
+# ------------------------------------------------------- latent decode step
+
+MLA_NAME = "mla_decode_b64_hq128_dqk576_dv512_ps64_ctx1k-8k"
+MLA_DESC = ("one latent (MLA) decode step, B=64 sequences, Hq=128 query heads sharing one latent "
+            "cache of 576 components (values: the first 512), page_size=64, context lengths uniform "
+            "in [1024, 8192] by seed, pages in random order")
+
+
+def mla_inputs():
+    import numpy as np
+    from paper_2609_04523_gb300 import workloads as W
+    lens = [int(x) for x in np.random.default_rng(2001).integers(1024, 8193, size=64)]
+    return W.make_mla_paged(lens, 128, 64, seed=2002, spare_pages=64)
+
+
+def cpu_oracle_mla(inp, n_seq: int | None = None):
+    """The oracle, as it stands, on the first n_seq sequences of the step (all
+    of them by default).  Returns (seconds, threads, bytes of the sample, o, lse)."""
+    import oracle
+    from paper_2609_04523_gb300 import workloads as W
+    n = inp.q.shape[0] if n_seq is None else n_seq
+    t0 = time.perf_counter()
+    o, lse = oracle.mla_decode(inp.q[:n], inp.cache, inp.page_table[:n], inp.seq_lens[:n],
+                               inp.scale, inp.dv)
+    secs = time.perf_counter() - t0
+    nbytes = W.mla_decode_bytes([int(x) for x in inp.seq_lens[:n]], inp.q.shape[1])
+    return secs, oracle.default_threads(), nbytes, o, lse
+
+
+def run_mla(args, rank: int, world: int, local_rank: int):
+    import numpy as np
+    import torch
+
+    from paper_2609_04523_gb300 import binding, mk_attn_check_status
+    from paper_2609_04523_gb300 import workloads as W
+    from paper_2609_04523_gb300.build import build_library
+
+    build_library()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    inp = mla_inputs()
+    lens = [int(x) for x in inp.seq_lens]
+    B, Hq, _ = inp.q.shape
+    nbytes = W.mla_decode_bytes(lens, Hq)
+    flops = W.mla_decode_flops(lens, Hq)
+    q, c, pt, sl = (t.to(dev) for t in (inp.q, inp.cache, inp.page_table, inp.seq_lens))
+    o = torch.empty((B, Hq, binding.MLA_DV), dtype=torch.bfloat16, device=dev)
+    lse = torch.empty((B, Hq), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    props = torch.cuda.get_device_properties(dev)
+    pci_bus_id = None
+    if hasattr(props, "pci_bus_id"):
+        pci_bus_id = "%08x:%02x:%02x.0" % (getattr(props, "pci_domain_id", 0), props.pci_bus_id,
+                                           getattr(props, "pci_device_id", 0))
+    need = binding.mk_attn_mla_decode_workspace_bytes(B, Hq, c.shape[1], pt.shape[1])
+    ws = torch.empty(max(need, 16) // 4, dtype=torch.float32, device=dev) if need > 0 else None
+    launches = 2 if need > 0 else 1
+
+    def step():
+        binding.mla_decode_paged(q, c, pt, sl, inp.scale, out=o, lse=lse, workspace=ws,
+                                 stream=stream)
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize(dev)
+    if mk_attn_check_status(stream.cuda_stream) != 0:
+        raise RuntimeError("latent decode kernel reported an error during warm-up")
+
+    def timed_region():
+        starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize(dev)
+        with ClockSampler(pci_bus_id, local_rank) as cs:
+            for i in range(args.steps):
+                flush.zero_()
+                starts[i].record(stream)
+                step()
+                ends[i].record(stream)
+            torch.cuda.synchronize(dev)
+        if world > 1:
+            torch.distributed.barrier()
+        return [a.elapsed_time(b) for a, b in zip(starts, ends)], cs.summary()
+
+    ms, clocks = timed_region()
+    remeasured = False
+    if clocks_rejected(clocks):
+        ms, clocks = timed_region()
+        remeasured = True
+    if mk_attn_check_status(stream.cuda_stream) != 0:
+        raise RuntimeError("latent decode kernel reported an error in the timed region")
+    total_ms = max_over_ranks(sum(ms), world, dev)
+    ms_per_step = total_ms / args.steps
+    gbs_job = world * nbytes * args.steps / (total_ms * 1e-3) / 1e9
+    gbs = nbytes / (ms_per_step * 1e-3) / 1e9
+    tflops = flops / (ms_per_step * 1e-3) / 1e12
+
+    # End to end: the latent cache stays on the device; each step copies the
+    # new queries, page table and lengths in and o, lse out.
+    qh, pth, slh = inp.q.pin_memory(), inp.page_table.pin_memory(), inp.seq_lens.pin_memory()
+    oh = torch.empty(o.shape, dtype=o.dtype).pin_memory()
+    lh = torch.empty(lse.shape, dtype=lse.dtype).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for t in (qh, pth, slh))
+    d2h = oh.numel() * oh.element_size() + lh.numel() * lh.element_size()
+    qd, ptd, sld = torch.empty_like(q), torch.empty_like(pt), torch.empty_like(sl)
+
+    def e2e_step():
+        qd.copy_(qh, non_blocking=True)
+        ptd.copy_(pth, non_blocking=True)
+        sld.copy_(slh, non_blocking=True)
+        binding.mla_decode_paged(qd, c, ptd, sld, inp.scale, out=o, lse=lse, workspace=ws,
+                                 stream=stream)
+        oh.copy_(o, non_blocking=True)
+        lh.copy_(lse, non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize(dev)
+    if world > 1:
+        torch.distributed.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    e2e_gbs = world * nbytes * args.steps / (e2e_ms * 1e-3) / 1e9
+
+    if rank != 0:
+        return None
+    peaks, peak_src = measured_peaks()
+    peak = float(peaks["hbm_gbs"])
+    line = {
+        "metric": MLA_METRIC,
+        "value": round(gbs_job, 1),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 5),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) bf16 queries and latent cache, seeded lengths and page order)",
+        "config": {
+            "workload": f"{MLA_NAME}: {MLA_DESC}",
+            "bytes_per_step_per_gpu": nbytes,
+            "byte_convention": "every cached latent row read once, q read, o and lse written",
+            "flops_per_step_per_gpu": flops,
+            "tflops": round(tflops, 2),
+            "flop_convention": "2 (576 + 512) per query head and cached key",
+            "cached_keys": sum(lens),
+            "l2": "flushed before every timed step (256 MiB device write, outside the event pair); "
+                  "the cache (%.2f GB) is larger than L2" % (2 * sum(lens) * 576 / 1e9),
+            "timing": "CUDA events around each call (latent decode kernel and, with several KV "
+                      "splits, the merge kernel) on the launching stream; sum over steps",
+            "parallelism": f"replicas x{world} (independent workloads per GPU)",
+        },
+        "roofline": {
+            "bound": "hbm",
+            "achieved": round(gbs, 1),
+            "peak": peak,
+            "unit": "GB/s",
+            "frac": round(gbs / peak, 4),
+            "traffic": ncu_traffic(MLA_NAME, MLA_SOURCES),
+            "peak_source": f"{peak_src} HBM copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
+            "kernel": "mk::mla::mla_decode_kernel" + (" + mla_merge_kernel" if need > 0 else ""),
+        },
+        "e2e": {"value": round(e2e_gbs, 1), "unit": "GB/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": args.steps * launches,
+        "clocks": clocks,
+    }
+    if remeasured:
+        line["clocks_note"] = "first timed region saw a rejected clock state; re-measured once"
+    if not args.no_cpu_baseline:
+        secs, cores, sbytes, o_ref, lse_ref = cpu_oracle_mla(inp)
+        line["cpu_baseline"] = {"value": round(sbytes / secs / 1e9, 3), "unit": "GB/s",
+                                "cores": cores, "kind": "oracle",
+                                "sample": f"the whole step, {secs:.1f} s on {cores} threads"}
+        d = o.float().cpu().double().numpy() - o_ref
+        line["parity_spot_check"] = {
+            "rows": int(B * Hq),
+            "o_max_abs": float(np.max(np.abs(d))),
+            "o_rel_rms": float(math.sqrt(np.sum(d * d) / np.sum(o_ref * o_ref))),
+            "lse_max_abs": float(np.max(np.abs(lse.double().cpu().numpy() - lse_ref))),
+        }
+    return line
+
+
+def run_mla_reference(args, rank: int):
+    """The oracle, as it stands, on the leading sequences of the step, as many
+    as fit a per-step time budget that keeps the run within a few minutes."""
+    if rank != 0:
+        return None
+    inp = mla_inputs()
+    budget = max(1.0, min(10.0, 150.0 / max(1, args.steps + args.warmup)))
+    secs1, _, _, _, _ = cpu_oracle_mla(inp, 1)
+    n_seq = int(max(1, min(inp.q.shape[0], budget / max(secs1, 1e-3))))
+    vals, cores, secs = [], None, 0.0
+    for i in range(args.warmup + args.steps):
+        secs, cores, sbytes, _, _ = cpu_oracle_mla(inp, n_seq)
+        if i >= args.warmup:
+            vals.append(sbytes / secs / 1e9)
+    value = statistics.median(vals)
+    return {
+        "impl": "reference", "metric": MLA_METRIC, "value": round(value, 3), "unit": "GB/s",
+        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": None,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded N(0,1) bf16 queries and latent cache)",
+        "config": {"workload": f"{MLA_NAME}: {MLA_DESC}",
+                   "note": "the fp64 CPU oracle, as it stands, on the leading sequences per step"},
+        "cpu_baseline": {"value": round(value, 3), "unit": "GB/s", "cores": cores, "kind": "oracle",
+                         "sample": f"per step: the first {n_seq} sequences, {secs:.1f} s"},
+        "e2e": {"value": round(value, 3), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+        "gpu_launches": 0,
+    }
+
+
 # ----------------------------------------------------------- reference arm
 
 def run_reference(args, rank: int):
@@ -971,6 +1206,8 @@ def main():
             line = run_decode_reference(args, rank)
         elif args.workload == "backward":
             line = run_backward_reference(args, rank)
+        elif args.workload == "mla":
+            line = run_mla_reference(args, rank)
         else:
             line = run_reference(args, rank)
         if line is not None:
@@ -985,6 +1222,8 @@ def main():
             line = run_decode(args, rank, world, local_rank)
         elif args.workload == "backward":
             line = run_backward(args, rank, world, local_rank)
+        elif args.workload == "mla":
+            line = run_mla(args, rank, world, local_rank)
         else:
             line = run_ours(args, rank, world, local_rank)
     finally:

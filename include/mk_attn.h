@@ -256,6 +256,57 @@ MK_API int mk_attn_decode_paged_noalloc(const void *q, const void *k_cache, cons
                                         int page_size, int max_pages, int num_pages, float scale,
                                         void *stream);
 
+/* Latent (MLA) decode: row width of the latent cache (512 latent + 64 rotary
+ * components) and of the values (the first 512 components). */
+#define MK_MLA_DQK 576
+#define MK_MLA_DV 512
+
+/*
+ * mk_attn_mla_decode_workspace_bytes -- bytes of device workspace that
+ * mk_attn_mla_decode_paged needs for these sizes on the current device (0:
+ * none), or -1 for invalid sizes.
+ */
+MK_API int64_t mk_attn_mla_decode_workspace_bytes(int B, int Hq, int page_size, int max_pages);
+
+/*
+ * mk_attn_mla_decode_paged -- one decode step of multi-head latent attention
+ * in its absorbed form (the paper's MLA Attention row, Table 2 and Table 3):
+ * every query head attends to one shared latent cache, whose rows are the
+ * keys in full (MK_MLA_DQK components) and the values through their first
+ * MK_MLA_DV components.  For sequence b and query head h:
+ *   o[b,h,:] = sum_j softmax_j(scale * q[b,h,:] . c_j) c_j[:MK_MLA_DV]
+ *   lse[b,h] = ln sum_j exp(scale * q[b,h,:] . c_j)
+ * over the L_b = seq_lens[b] cached positions, position j being slot
+ * j % page_size of page page_table[b, j / page_size].
+ *
+ * Arguments (all pointers are DEVICE pointers owned by the caller):
+ *   q           bf16 [B, Hq, MK_MLA_DQK].  Read only.
+ *   cache       bf16 [num_pages, page_size, MK_MLA_DQK].  Read only.  Slots
+ *               of a sequence's last page past L_b are read (with weight
+ *               zero) and must hold finite values.
+ *   page_table  int32 [B, max_pages]; entries j < ceil(L_b / page_size) in
+ *               [0, num_pages).  seq_lens int32 [B], each in
+ *               [0, max_pages * page_size].
+ *   o           bf16 [B, Hq, MK_MLA_DV] output; lse fp32 [B, Hq] output
+ *               (natural log, scale included); L_b = 0 gives o = 0 and
+ *               lse = -inf.
+ *   Hq          any (groups of 128 heads), B * ceil(Hq / 128) <= 65535.
+ *   page_size   16, 32, 64 or 128.
+ *   workspace   device buffer of at least mk_attn_mla_decode_workspace_bytes()
+ *               bytes, 16-byte aligned, or NULL when that is 0 (scratch for
+ *               the per-split partials; calls sharing it must not overlap).
+ *   stream      cudaStream_t; asynchronous, never synchronises.
+ * Returns MK_OK, MK_ERR_INVALID_ARG, MK_ERR_UNSUPPORTED (page_size, grid
+ * limits), MK_ERR_ALIGNMENT (q, cache, o, workspace not 16-byte aligned;
+ * page_table, seq_lens, lse not 4-byte aligned) or MK_ERR_CUDA; on any
+ * error nothing is launched.  Device-side inputs out of range make the next
+ * mk_attn_check_status return MK_ERR_INVALID_ARG.
+ */
+MK_API int mk_attn_mla_decode_paged(const void *q, const void *cache, const int32_t *page_table,
+                                    const int32_t *seq_lens, void *o, float *lse, int B, int Hq,
+                                    int page_size, int max_pages, int num_pages, float scale,
+                                    void *workspace, int64_t workspace_bytes, void *stream);
+
 /* Schedules of work units over the persistent CTAs (mk_attn_tuning.schedule).
  * Units are numbered heaviest first (causal: the query tiles that see the most
  * keys, or the key tiles seen by the most queries). */

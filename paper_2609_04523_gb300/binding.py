@@ -24,6 +24,9 @@ MK_ERR_SCRATCH_LIMIT = -6
 # Backward-pass stages (MK_BWD_* in include/mk_attn.h).
 BWD_DELTA, BWD_DKDV, BWD_DQ, BWD_ALL = 1, 2, 4, 7
 
+# Latent (MLA) decode row widths (MK_MLA_DQK, MK_MLA_DV).
+MLA_DQK, MLA_DV = 576, 512
+
 # Unit schedules (MK_SCHED_*).
 SCHED_SNAKE, SCHED_ROUND_ROBIN, SCHED_BLOCKED = 0, 1, 2
 
@@ -50,7 +53,7 @@ EXPORTED = ("mk_attn_fwd", "mk_attn_fwd_stall_test", "mk_attn_bwd_workspace_byte
             "mk_attn_decode_workspace_bytes",
             "mk_attn_decode_paged", "mk_attn_decode_paged_noalloc", "mk_attn_error_string",
             "mk_attn_check_status", "mk_attn_version", "mk_attn_set_tuning",
-            "mk_attn_get_tuning")
+            "mk_attn_get_tuning", "mk_attn_mla_decode_workspace_bytes", "mk_attn_mla_decode_paged")
 
 _lock = threading.Lock()
 _lib = None
@@ -104,6 +107,11 @@ def load_library() -> ctypes.CDLL:
             lib.mk_attn_check_status.restype = i
             lib.mk_attn_version.argtypes = []
             lib.mk_attn_version.restype = i
+            lib.mk_attn_mla_decode_workspace_bytes.argtypes = [i, i, i, i]
+            lib.mk_attn_mla_decode_workspace_bytes.restype = i64
+            lib.mk_attn_mla_decode_paged.argtypes = [vp, vp, vp, vp, vp, vp, i, i, i, i, i,
+                                                     ctypes.c_float, vp, i64, vp]
+            lib.mk_attn_mla_decode_paged.restype = i
             lib.mk_attn_set_tuning.argtypes = [ctypes.POINTER(MkAttnTuning)]
             lib.mk_attn_set_tuning.restype = i
             lib.mk_attn_get_tuning.argtypes = [ctypes.POINTER(MkAttnTuning)]
@@ -384,4 +392,63 @@ def decode_paged(q, k_cache, v_cache, page_table, seq_lens, scale: float | None 
                                 page_table.data_ptr(), seq_lens.data_ptr(), out.data_ptr(),
                                 lse.data_ptr(), B, Hq, Hkv, D, page_size, max_pages, num_pages,
                                 float(scale), ws_ptr, ws_bytes, stream.cuda_stream))
+    return out, lse
+
+
+def mk_attn_mla_decode_workspace_bytes(B: int, Hq: int, page_size: int, max_pages: int) -> int:
+    return load_library().mk_attn_mla_decode_workspace_bytes(B, Hq, page_size, max_pages)
+
+
+def mk_attn_mla_decode_paged(q: int, cache: int, page_table: int, seq_lens: int, o: int, lse: int,
+                             B: int, Hq: int, page_size: int, max_pages: int, num_pages: int,
+                             scale: float, workspace: int | None, workspace_bytes: int,
+                             stream: int | None) -> int:
+    """Raw C-ABI call: integer device pointers in, status code out."""
+    return load_library().mk_attn_mla_decode_paged(q, cache, page_table, seq_lens, o, lse, B, Hq,
+                                                   page_size, max_pages, num_pages, float(scale),
+                                                   workspace, int(workspace_bytes), stream)
+
+
+def mla_decode_paged(q, cache, page_table, seq_lens, scale: float | None = None, out=None,
+                     lse=None, workspace=None, stream=None):
+    """One latent (MLA) decode step through mk_attn_mla_decode_paged.
+
+    q: [B, Hq, 576] bf16; cache: [num_pages, page_size, 576] bf16 (keys in
+    full, values = the first 512 components); page_table: int32 [B,
+    max_pages]; seq_lens: int32 [B]; all CUDA tensors.  Returns (o [B, Hq,
+    512] bf16, lse [B, Hq] fp32).  The fp32 split workspace is allocated here
+    unless one is passed."""
+    import torch
+    for name, t in (("q", q), ("cache", cache)):
+        if not t.is_cuda or t.dtype != torch.bfloat16 or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous bf16 CUDA tensor")
+    for name, t in (("page_table", page_table), ("seq_lens", seq_lens)):
+        if not t.is_cuda or t.dtype != torch.int32 or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous int32 CUDA tensor")
+    if q.dim() != 3 or q.shape[2] != MLA_DQK or cache.dim() != 3 or cache.shape[2] != MLA_DQK:
+        raise ValueError(f"q [B, Hq, {MLA_DQK}], cache [num_pages, page_size, {MLA_DQK}]")
+    B, Hq, _ = q.shape
+    num_pages, page_size, _ = cache.shape
+    if page_table.dim() != 2 or page_table.shape[0] != B or seq_lens.shape != (B,):
+        raise ValueError("page_table [B, max_pages], seq_lens [B]")
+    max_pages = page_table.shape[1]
+    if scale is None:
+        scale = 1.0 / float(MLA_DQK) ** 0.5
+    if out is None:
+        out = torch.empty((B, Hq, MLA_DV), dtype=torch.bfloat16, device=q.device)
+    if lse is None:
+        lse = torch.empty((B, Hq), dtype=torch.float32, device=q.device)
+    need = mk_attn_mla_decode_workspace_bytes(B, Hq, page_size, max_pages)
+    if need < 0:
+        raise MkAttnError(MK_ERR_INVALID_ARG, "invalid MLA decode sizes")
+    if workspace is None and need > 0:
+        workspace = torch.empty((need + 15) // 16 * 4, dtype=torch.float32, device=q.device)
+    ws_ptr = None if workspace is None else workspace.data_ptr()
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    if stream is None:
+        stream = torch.cuda.current_stream(q.device)
+    _check(mk_attn_mla_decode_paged(q.data_ptr(), cache.data_ptr(), page_table.data_ptr(),
+                                    seq_lens.data_ptr(), out.data_ptr(), lse.data_ptr(), B, Hq,
+                                    page_size, max_pages, num_pages, float(scale), ws_ptr,
+                                    ws_bytes, stream.cuda_stream))
     return out, lse

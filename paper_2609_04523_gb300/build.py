@@ -18,7 +18,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB_NAME = "libmk_attn.so"
 LIB_PATH = os.path.join(PKG, LIB_NAME)
-SOURCES = [os.path.join(CSRC, f) for f in ("fmha_fwd.cu", "fmha_bwd.cu", "decode.cu", "status.cu")]
+SOURCES = [os.path.join(CSRC, f) for f in ("fmha_fwd.cu", "fmha_bwd.cu", "decode.cu", "mla_decode.cu", "status.cu")]
 DEPENDS = SOURCES + [os.path.join(CSRC, "ptx.cuh"), os.path.join(CSRC, "tma_host.h"),
                      os.path.join(INCLUDE, "mk_attn.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

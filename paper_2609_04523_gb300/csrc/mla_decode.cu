@@ -1,0 +1,637 @@
+// mla_decode.cu -- one decode step of multi-head latent attention (the
+// absorbed form) against a paged latent cache, for GB300 (sm_103a), and its C
+// ABI.
+//
+// Every query head attends to one shared latent cache: the cached row c_j
+// (576 = 512 latent + 64 rotary components) is the key in full and, through
+// its first 512 components, the value -- the paper's MLA Attention row
+// (Table 2, Table 3), under the contract of Sections 2.1 and 3.1:
+//   o[b,h,:512] = sum_j softmax_j(scale * q[b,h,:] . c_j) c_j[:512]
+//   lse[b,h]    = ln sum_j exp(scale * q[b,h,:] . c_j)
+// with position j in slot j % page_size of page page_table[b, j / page_size].
+//
+// All heads share every key, so the step is a pair of dense contractions per
+// block of 128 keys and runs on tcgen05 with the query heads as the MMA's M
+// dimension (up to 128 heads per CTA, missing heads zero-filled by TMA):
+//   S  = Q C^T        M = heads, N = 128 keys, K = 576 (nine 64-wide chunks)
+//   O += P C[:, :dv]  M = heads, N = 64 value components per MMA, K = 128 keys
+// Capacity sets the shape.  Q (128 x 576 bf16 = 144 KB) stays in shared
+// memory; the cache streams through a ring of five 16 KB chunk slots (128
+// keys x 64 components each), in the order the MMAs consume them: the nine
+// key chunks of block n+1, then the value chunks of block n (the same rows,
+// read again from L2).  O for 128 heads x 512 components would fill TMEM's
+// 512 columns, so the value dimension is split over two CTAs (each computes
+// S itself and keeps a 256-column O); TMEM is S double-buffered (2 x 128
+// columns) + O (256 columns).  Softmax: base 2, one thread per head row, the
+// lazy rescale of the forward kernel (O in TMEM is rescaled only when the
+// row max rises by more than 8); P (bf16) overwrites the first 64 columns of
+// its S buffer and is the TMEM A operand of the P.V MMAs.  KV splits with a
+// log-sum-exp merge fill the GPU at small batch, as in the paged decode step.
+//
+// Roles: warps 0-3 softmax and epilogue (thread = head row = TMEM lane),
+// warp 4 tcgen05 MMA issuer, warp 5 TMA producer.  One CTA per SM (shared
+// memory), persistent only within its split.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include <cmath>
+#include <cstdint>
+#include <mutex>
+
+#include "mk_attn.h"
+#include "ptx.cuh"
+#include "tma_host.h"
+
+namespace mk {
+namespace mla {
+
+constexpr int kDqk = MK_MLA_DQK;          // 576
+constexpr int kDv = MK_MLA_DV;            // 512
+constexpr int kChunk = 64;                // components per chunk (one 128-byte swizzle row)
+constexpr int kChunksK = kDqk / kChunk;   // 9
+constexpr int kDvCta = kDv / 2;           // 256 value components per CTA
+constexpr int kChunksV = kDvCta / kChunk; // 4
+constexpr int kHeads = 128;               // M: heads per CTA
+constexpr int kBlock = 128;               // keys per block (N of S)
+constexpr int kChunkBytes = kBlock * kChunk * 2;  // 16 KB: 128 rows x 128 B
+constexpr int kQBytes = kChunksK * kHeads * kChunk * 2;  // 144 KB
+constexpr int kSlots = 5;
+constexpr int kOffRing = kQBytes;
+constexpr int kOffCtl = kOffRing + kSlots * kChunkBytes;
+constexpr int kSmemBytes = kOffCtl + 256 + 1024;
+static_assert(kSmemBytes <= 232448, "shared memory per CTA");
+constexpr int kThreads = 192;
+constexpr int kMmaWarp = 4, kLoadWarp = 5;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kColS = 0;      // S buffer X at kColS + 128 X
+constexpr uint32_t kColO = 256;    // O: 256 columns
+constexpr float kRescaleThreshold = 8.0f;
+constexpr int kSplitCtasPerSm = 2;  // split planning: about two waves of CTAs
+
+__device__ int g_status = 0;
+
+struct Ctl {
+  uint64_t q_full;
+  uint64_t slot_full[kSlots], slot_empty[kSlots];
+  uint64_t s_full[2], p_full[2], pv_done[2];
+  uint64_t mma_drained;
+  uint32_t tmem_base;
+  int abort;
+};
+static_assert(sizeof(Ctl) <= 256, "control block");
+
+struct Params {
+  const int32_t *page_table;  // [B, max_pages]
+  const int32_t *seq_lens;    // [B]
+  uint16_t *o;                // bf16 [B, Hq, 512]
+  float *lse;                 // [B, Hq]
+  float *part;                // [B, Hq, n_splits, 516]: 512 components, lse, 3 pad; n_splits > 1
+  int B, Hq, head_groups;
+  int page_size, max_pages, num_pages;
+  int n_splits, blocks_per_split;
+  float scale_log2;
+};
+
+__device__ __forceinline__ void record(int status) { atomicCAS(&g_status, 0, status); }
+
+// The chunks a CTA consumes, in order: for block n, the nine key chunks of
+// block n (n < nb), then the four value chunks of block n - 1 (n >= 1); the
+// value chunks of the last block close the sequence.  Step t of that order:
+// which block and which chunk (component offset / 64).
+__device__ __forceinline__ void chunk_of_step(int t, int nb, int half, int &blk, int &chunk) {
+  // Steps per block n >= 1: 9 + 4 = 13; block 0 contributes 9.
+  if (t < kChunksK) {
+    blk = 0;
+    chunk = t;
+    return;
+  }
+  const int u = t - kChunksK;
+  const int n = 1 + u / (kChunksK + kChunksV);
+  const int r = u % (kChunksK + kChunksV);
+  if (n < nb) {
+    if (r < kChunksK) {
+      blk = n;
+      chunk = r;
+    } else {
+      blk = n - 1;
+      chunk = half * kChunksV + (r - kChunksK);
+    }
+  } else {  // n == nb: the closing value chunks of block nb - 1
+    blk = nb - 1;
+    chunk = half * kChunksV + r;
+  }
+}
+
+__device__ __forceinline__ void drain_wait(uint64_t *bar, uint32_t parity) {
+  int local_abort = 0;
+  mbar_wait(bar, parity, &local_abort);
+}
+
+// 2-D tiled TMA load (cache viewed as [tokens, 576]).
+__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, uint64_t *bar,
+                                            int32_t c0, int32_t c1, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_addr(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_addr(bar)), "r"(c0), "r"(c1), "l"(policy)
+      : "memory");
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    mla_decode_kernel(const __grid_constant__ CUtensorMap tm_q,
+                      const __grid_constant__ CUtensorMap tm_c, const Params p) {
+  const int split = blockIdx.x, half = blockIdx.y;
+  const int b = blockIdx.z / p.head_groups, hg = blockIdx.z % p.head_groups;
+  const int PS = p.page_size;
+  int L = p.seq_lens[b];
+  if (L < 0 || L > p.max_pages * PS) {
+    if (threadIdx.x == 0) record(MK_ERR_INVALID_ARG);
+    L = L < 0 ? 0 : p.max_pages * PS;
+  }
+  const int nblk_seq = (L + kBlock - 1) / kBlock;
+  const int first = split * p.blocks_per_split;
+  const int nb = max(0, min(first + p.blocks_per_split, nblk_seq) - first);
+  // Splits past the end of the sequence do nothing (the merge skips them);
+  // split 0 always runs, so an empty sequence still gets o = 0, lse = -inf.
+  if (split > 0 && nb == 0) return;
+
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw_addr = smem_addr(smem_raw);
+  uint8_t *smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);
+  Ctl *ctl = reinterpret_cast<Ctl *>(smem + kOffCtl);
+  const int warp = threadIdx.x / 32;
+
+  if (threadIdx.x == 0) {
+    mbar_init(&ctl->q_full, 1);
+    for (int s = 0; s < kSlots; ++s) {
+      mbar_init(&ctl->slot_full[s], 1);
+      mbar_init(&ctl->slot_empty[s], 1);
+    }
+    for (int x = 0; x < 2; ++x) {
+      mbar_init(&ctl->s_full[x], 1);
+      mbar_init(&ctl->p_full[x], kHeads);
+      mbar_init(&ctl->pv_done[x], 1);
+    }
+    mbar_init(&ctl->mma_drained, 1);
+    ctl->abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == kMmaWarp) {
+    tmem_alloc(&ctl->tmem_base, kTmemCols);
+    tmem_relinquish_alloc_permit();
+  }
+  tc_fence_before_sync();
+  __syncthreads();
+  tc_fence_after_sync();
+  const uint32_t tmem = ctl->tmem_base;
+  volatile int *abort = &ctl->abort;
+  const int n_steps = nb == 0 ? 0 : kChunksK + (nb - 1) * (kChunksK + kChunksV) + kChunksV;
+
+  if (warp == kLoadWarp) {
+    // ------------------------------------------------------------ producer
+    bool ok = true;
+    if (nb > 0) {
+      if (elect_one()) {
+        tma_prefetch_desc(&tm_q);
+        tma_prefetch_desc(&tm_c);
+        mbar_arrive_expect_tx(&ctl->q_full, kQBytes);
+        const uint64_t pol_q = l2_policy_evict_last();  // both value halves read it
+#pragma unroll 1
+        for (int c = 0; c < kChunksK; ++c)
+          tma_load_3d(smem + c * kHeads * kChunk * 2, &tm_q, &ctl->q_full, c * kChunk,
+                      hg * kHeads, b, pol_q);
+      }
+      __syncwarp();
+    }
+    const uint64_t pol_c = l2_policy_evict_last();  // read again for the values
+    const int pages_per_block = kBlock / PS;
+    for (int t = 0; ok && t < n_steps; ++t) {
+      const int s = t % kSlots;
+      ok = mbar_wait_all(&ctl->slot_empty[s], ((t / kSlots) & 1) ^ 1, abort);
+      if (!ok) break;
+      if (elect_one()) {
+        int blk, chunk;
+        chunk_of_step(t, nb, half, blk, chunk);
+        const int page0 = (first + blk) * pages_per_block;  // logical page of the block's row 0
+        const int n_pages_seq = (L + PS - 1) / PS;
+        mbar_arrive_expect_tx(&ctl->slot_full[s], kChunkBytes);
+        uint8_t *dst = smem + kOffRing + s * kChunkBytes;
+        for (int i = 0; i < pages_per_block; ++i) {
+          // Pages past the sequence end load its first page of the block
+          // instead (finite rows, masked out), so the byte count holds.
+          const int lp = page0 + i < n_pages_seq ? page0 + i : page0;
+          int page = p.page_table[(int64_t)b * p.max_pages + lp];
+          if (page < 0 || page >= p.num_pages) {
+            record(MK_ERR_INVALID_ARG);
+            page = 0;
+          }
+          tma_load_2d(dst + i * PS * 128, &tm_c, &ctl->slot_full[s], chunk * kChunk, page * PS,
+                      pol_c);
+        }
+      }
+      __syncwarp();
+    }
+    // Teardown: the loads issued land before the CTA exits.
+    if (nb > 0) drain_wait(&ctl->q_full, 0);
+    for (int t = max(0, n_steps - kSlots); t < n_steps; ++t)
+      drain_wait(&ctl->slot_full[t % kSlots], (t / kSlots) & 1);
+  } else if (warp == kMmaWarp) {
+    // ---------------------------------------------------------- MMA issuer
+    constexpr uint32_t idesc_s = idesc_bf16_f32(kHeads, kBlock, false, false);
+    constexpr uint32_t idesc_pv = idesc_bf16_f32(kHeads, kChunk, false, true);
+    const uint32_t sQ = smem_addr(smem);
+    const uint32_t sRing = smem_addr(smem + kOffRing);
+    bool ok = true;
+    int t = 0;  // chunk step
+    auto take_slot = [&]() -> uint32_t {
+      const int s = t % kSlots;
+      ok = mbar_wait_all(&ctl->slot_full[s], (t / kSlots) & 1, abort);
+      tc_fence_after_sync();
+      return sRing + s * kChunkBytes;
+    };
+    auto release_slot = [&]() {
+      if (elect_one()) umma_commit(&ctl->slot_empty[t % kSlots]);
+      __syncwarp();
+      ++t;
+    };
+    // S(x) = Q C_n^T over the nine key chunks of block n.
+    auto issue_s = [&](int x) {
+      for (int c = 0; ok && c < kChunksK; ++c) {
+        const uint32_t kaddr = take_slot();
+        if (!ok) break;
+        if (elect_one()) {
+          const uint64_t a0 = sdesc_sw128(sQ + c * kHeads * kChunk * 2, 16, 1024);
+          const uint64_t b0 = sdesc_sw128(kaddr, 16, 1024);
+#pragma unroll
+          for (int kk = 0; kk < kChunk / 16; ++kk)
+            umma_ss(tmem + kColS + x * 128, a0 + kk * 2, b0 + kk * 2, idesc_s,
+                    (c > 0 || kk > 0) ? 1u : 0u);
+        }
+        __syncwarp();
+        release_slot();
+      }
+      if (ok && elect_one()) umma_commit(&ctl->s_full[x]);
+      __syncwarp();
+    };
+    // O (+)= P(x) C_n[:, value chunks of this CTA]: P is bf16 in the first 64
+    // columns of S buffer x (the TMEM A operand), each value chunk an
+    // MN-major B operand of 128 keys x 64 components.
+    auto issue_pv = [&](int x, bool first_block) {
+      for (int cv = 0; ok && cv < kChunksV; ++cv) {
+        const uint32_t vaddr = take_slot();
+        if (!ok) break;
+        if (elect_one()) {
+          const uint64_t b0 = sdesc_sw128(vaddr, 1024, 1024);
+#pragma unroll
+          for (int kk = 0; kk < kBlock / 16; ++kk)
+            umma_ts(tmem + kColO + cv * kChunk, tmem + kColS + x * 128 + kk * 8,
+                    b0 + (uint64_t)(kk * 128), idesc_pv, (!first_block || kk > 0) ? 1u : 0u);
+        }
+        __syncwarp();
+        release_slot();
+      }
+    };
+    if (nb > 0) {
+      ok = mbar_wait_all(&ctl->q_full, 0, abort);
+      if (ok) issue_s(0);
+      for (int n = 0; ok && n < nb; ++n) {
+        // S(n+1) into the other buffer: its P(n-1) was read by PV(n-1),
+        // issued before this.
+        if (n + 1 < nb) issue_s((n + 1) & 1);
+        if (!ok) break;
+        ok = mbar_wait_all(&ctl->p_full[n & 1], (n >> 1) & 1, abort);
+        if (!ok) break;
+        tc_fence_after_sync();
+        issue_pv(n & 1, n == 0);
+        if (ok && elect_one()) umma_commit(&ctl->pv_done[n & 1]);
+        __syncwarp();
+      }
+    }
+    if (elect_one()) umma_commit(&ctl->mma_drained);
+    __syncwarp();
+    drain_wait(&ctl->mma_drained, 0);
+  } else {
+    // ------------------------------------------------------------ softmax
+    const int row = threadIdx.x;  // head within the group = TMEM lane
+    const uint32_t t_row = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+    const float c2 = p.scale_log2;
+    float m_run = -INFINITY, l_run = 0.f;
+    bool ok = true;
+    for (int n = 0; ok && n < nb; ++n) {
+      const int x = n & 1;
+      ok = mbar_wait_all(&ctl->s_full[x], (n >> 1) & 1, abort);
+      if (!ok) break;
+      tc_fence_after_sync();
+      float s[kBlock];
+      {
+        uint32_t raw[4][32];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) tmem_ld_32x32b_x32(t_row + kColS + x * 128 + c * 32, raw[c]);
+        tmem_ld_wait();
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          reg_fence(raw[c]);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) s[c * 32 + e] = __uint_as_float(raw[c][e]) * c2;
+        }
+      }
+      const int key0 = (first + n) * kBlock;
+      if (key0 + kBlock > L) {
+#pragma unroll
+        for (int c = 0; c < kBlock; ++c) s[c] = key0 + c < L ? s[c] : -INFINITY;
+      }
+      float mx0 = fmaxf(s[0], s[1]), mx1 = fmaxf(s[2], s[3]);
+      float mx2 = fmaxf(s[4], s[5]), mx3 = fmaxf(s[6], s[7]);
+#pragma unroll
+      for (int c = 8; c < kBlock; c += 8) {
+        mx0 = fmax3(mx0, s[c], s[c + 1]);
+        mx1 = fmax3(mx1, s[c + 2], s[c + 3]);
+        mx2 = fmax3(mx2, s[c + 4], s[c + 5]);
+        mx3 = fmax3(mx3, s[c + 6], s[c + 7]);
+      }
+      const float m_new = fmaxf(m_run, fmaxf(fmax3(mx0, mx1, mx2), mx3));
+      if (m_new > m_run + kRescaleThreshold) {
+        const float alpha = ex2_approx(m_run - m_new);  // 0 when m_run = -inf
+        l_run *= alpha;
+        m_run = m_new;
+        if (n > 0) {
+          // O holds blocks 0..n-1 once PV(n-1) is done (PV(n-2) is, since
+          // S(n) was issued after it).
+          ok = mbar_wait_all(&ctl->pv_done[(n - 1) & 1], ((n - 1) >> 1) & 1, abort);
+          if (!ok) break;
+          tc_fence_after_sync();
+#pragma unroll 1
+          for (int c = 0; c < kDvCta / 32; ++c) {
+            uint32_t o_raw[32];
+            tmem_ld_32x32b_x32(t_row + kColO + c * 32, o_raw);
+            tmem_ld_wait();
+            reg_fence(o_raw);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) o_raw[e] = __float_as_uint(__uint_as_float(o_raw[e]) * alpha);
+            tmem_st_32x32b_x32(t_row + kColO + c * 32, o_raw);
+          }
+          tmem_st_wait();
+        }
+      }
+      const float neg_m = m_run == -INFINITY ? 0.f : -m_run;
+      float sum0 = 0.f, sum1 = 0.f, sum2 = 0.f, sum3 = 0.f;
+      uint32_t pk[2][32];
+#pragma unroll
+      for (int c = 0; c < kBlock; c += 4) {
+        const float p0 = ex2_approx(s[c] + neg_m), p1 = ex2_approx(s[c + 1] + neg_m);
+        const float p2 = ex2_approx(s[c + 2] + neg_m), p3 = ex2_approx(s[c + 3] + neg_m);
+        fadd2_acc(sum0, sum1, p0, p1);
+        fadd2_acc(sum2, sum3, p2, p3);
+        pk[c / 64][(c % 64) / 2] = pack_bf16x2(p0, p1);
+        pk[c / 64][(c % 64) / 2 + 1] = pack_bf16x2(p2, p3);
+      }
+      l_run += (sum0 + sum1) + (sum2 + sum3);
+      tmem_st_32x32b_x32(t_row + kColS + x * 128, pk[0]);
+      tmem_st_32x32b_x32(t_row + kColS + x * 128 + 32, pk[1]);
+      tmem_st_wait();
+      tc_fence_before_sync();
+      mbar_arrive(&ctl->p_full[x]);
+    }
+    // ------------------------------------------------------------ epilogue
+    if (ok && nb > 0) {
+      // PV(nb-1) and PV(nb-2) done: each pv_done buffer has no later phase.
+      ok = mbar_wait_all(&ctl->pv_done[(nb - 1) & 1], ((nb - 1) >> 1) & 1, abort);
+      if (ok && nb > 1) ok = mbar_wait_all(&ctl->pv_done[(nb - 2) & 1], ((nb - 2) >> 1) & 1, abort);
+      tc_fence_after_sync();
+    }
+    const int h = hg * kHeads + row;
+    if (ok) {
+      const bool valid = h < p.Hq;
+      const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
+      const float lse = l_run > 0.f ? (m_run + log2f(l_run)) * 0.69314718055994530942f : -INFINITY;
+      const int64_t bh = (int64_t)b * p.Hq + h;
+#pragma unroll 1
+      for (int c = 0; c < kDvCta / 32; ++c) {
+        float v[32];
+        if (nb > 0) {
+          uint32_t o_raw[32];
+          tmem_ld_32x32b_x32(t_row + kColO + c * 32, o_raw);
+          tmem_ld_wait();
+          reg_fence(o_raw);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) v[e] = __uint_as_float(o_raw[e]) * inv_l;
+        } else {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) v[e] = 0.f;
+        }
+        if (!valid) continue;
+        const int d0 = half * kDvCta + c * 32;
+        if (p.n_splits == 1) {
+          uint4 *dst = reinterpret_cast<uint4 *>(p.o + bh * kDv + d0);
+#pragma unroll
+          for (int e = 0; e < 4; ++e)
+            dst[e] = make_uint4(pack_bf16x2(v[8 * e], v[8 * e + 1]), pack_bf16x2(v[8 * e + 2], v[8 * e + 3]),
+                                pack_bf16x2(v[8 * e + 4], v[8 * e + 5]), pack_bf16x2(v[8 * e + 6], v[8 * e + 7]));
+        } else {
+          float4 *dst = reinterpret_cast<float4 *>(p.part + (bh * p.n_splits + split) * (kDv + 4) + d0);
+#pragma unroll
+          for (int e = 0; e < 8; ++e) dst[e] = make_float4(v[4 * e], v[4 * e + 1], v[4 * e + 2], v[4 * e + 3]);
+        }
+      }
+      if (valid && half == 0) {
+        if (p.n_splits == 1)
+          p.lse[bh] = lse;
+        else
+          p.part[(bh * p.n_splits + split) * (kDv + 4) + kDv] = lse;
+      }
+    }
+    if (!ok) *abort = 1;
+  }
+
+  tc_fence_before_sync();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    tc_fence_after_sync();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+  if (threadIdx.x == 0 && ctl->abort) record(MK_ERR_TIMEOUT);
+}
+
+// Combines the splits of each (b, h) by their log-sum-exps (as the paged
+// decode step's merge), one warp per (b, h): each split's partial is
+// o_s = (sum over its keys of exp(s_j) c_j) / exp(lse_s), stored with lse_s
+// at component 512 of a 516-float row.
+__global__ void __launch_bounds__(128) mla_merge_kernel(const Params p) {
+  constexpr int NDL = kDv / 32;
+  const int row = blockIdx.x * 4 + threadIdx.x / 32;  // b * Hq + h
+  if (row >= p.B * p.Hq) return;
+  const int lane = lane_id();
+  const float *pr = p.part + (int64_t)row * p.n_splits * (kDv + 4);
+  int L = p.seq_lens[row / p.Hq];
+  L = L < 0 ? 0 : (L > p.max_pages * p.page_size ? p.max_pages * p.page_size : L);
+  const int nblk = (L + kBlock - 1) / kBlock;
+  const int n_valid = max(1, min(p.n_splits, (nblk + p.blocks_per_split - 1) / p.blocks_per_split));
+  float mx = -INFINITY;
+  for (int s = 0; s < n_valid; ++s) mx = fmaxf(mx, pr[s * (kDv + 4) + kDv]);
+  float acc[NDL];
+#pragma unroll
+  for (int e = 0; e < NDL; ++e) acc[e] = 0.f;
+  float wsum = 0.f;
+  if (mx > -INFINITY) {
+    for (int s = 0; s < n_valid; ++s) {
+      const float w = exp2f((pr[s * (kDv + 4) + kDv] - mx) * 1.4426950408889634f);
+      wsum += w;
+      const float4 *src = reinterpret_cast<const float4 *>(pr + s * (kDv + 4) + lane * NDL);
+#pragma unroll
+      for (int e = 0; e < NDL / 4; ++e) {
+        const float4 f = src[e];
+        acc[4 * e] = fmaf(w, f.x, acc[4 * e]);
+        acc[4 * e + 1] = fmaf(w, f.y, acc[4 * e + 1]);
+        acc[4 * e + 2] = fmaf(w, f.z, acc[4 * e + 2]);
+        acc[4 * e + 3] = fmaf(w, f.w, acc[4 * e + 3]);
+      }
+    }
+  }
+  const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
+  uint4 *orow = reinterpret_cast<uint4 *>(p.o + (int64_t)row * kDv + lane * NDL);
+#pragma unroll
+  for (int e = 0; e < NDL / 8; ++e)
+    orow[e] = make_uint4(pack_bf16x2(acc[8 * e] * inv, acc[8 * e + 1] * inv),
+                         pack_bf16x2(acc[8 * e + 2] * inv, acc[8 * e + 3] * inv),
+                         pack_bf16x2(acc[8 * e + 4] * inv, acc[8 * e + 5] * inv),
+                         pack_bf16x2(acc[8 * e + 6] * inv, acc[8 * e + 7] * inv));
+  if (lane == 0) p.lse[row] = wsum > 0.f ? mx + logf(wsum) : -INFINITY;
+}
+
+// ------------------------------------------------------------------- host
+
+struct DeviceInfo {
+  std::once_flag once;
+  int sm_count = 0;
+  cudaError_t attr = cudaSuccess;
+};
+static DeviceInfo g_devices[64];
+
+static int sm_count_and_setup() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  DeviceInfo &di = g_devices[dev];
+  std::call_once(di.once, [&] {
+    if (cudaDeviceGetAttribute(&di.sm_count, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      di.sm_count = 0;
+    di.attr = cudaFuncSetAttribute(mla_decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   kSmemBytes);
+  });
+  return di.attr == cudaSuccess ? di.sm_count : 0;
+}
+
+// KV splits of whole 128-key blocks: about kSplitCtasPerSm CTAs per SM over
+// B x head groups x 2 value halves.
+static void plan(int B, int head_groups, int max_blocks, int sms, int &n_splits, int &bps) {
+  const int64_t units = (int64_t)B * head_groups * 2;
+  int64_t want = ((int64_t)kSplitCtasPerSm * sms + units - 1) / units;
+  want = want < 1 ? 1 : (want > max_blocks ? max_blocks : want);
+  bps = (int)((max_blocks + want - 1) / want);
+  n_splits = (max_blocks + bps - 1) / bps;
+}
+
+static bool encode(CUtensorMap *map, const void *base, int rank, const cuuint64_t *dims,
+                   const cuuint64_t *strides, const cuuint32_t *box) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return false;
+  const cuuint32_t estr[3] = {1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void *>(base), dims, strides,
+             box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace mla
+
+int mla_take_status() {
+  int h = 0;
+  if (cudaMemcpyFromSymbol(&h, mla::g_status, sizeof(int)) != cudaSuccess) return MK_ERR_CUDA;
+  if (h != 0) {
+    const int zero = 0;
+    if (cudaMemcpyToSymbol(mla::g_status, &zero, sizeof(int)) != cudaSuccess) return MK_ERR_CUDA;
+  }
+  return h;
+}
+
+}  // namespace mk
+
+extern "C" {
+
+int64_t mk_attn_mla_decode_workspace_bytes(int B, int Hq, int page_size, int max_pages) {
+  if (B < 1 || Hq < 1 || page_size < 1 || max_pages < 1) return -1;
+  const int sms = mk::mla::sm_count_and_setup();
+  if (sms <= 0) return -1;
+  const int64_t max_keys = (int64_t)max_pages * page_size;
+  const int max_blocks = (int)((max_keys + mk::mla::kBlock - 1) / mk::mla::kBlock);
+  const int head_groups = (Hq + mk::mla::kHeads - 1) / mk::mla::kHeads;
+  int n_splits = 1, bps = max_blocks;
+  mk::mla::plan(B, head_groups, max_blocks, sms, n_splits, bps);
+  if (n_splits == 1) return 0;
+  return (int64_t)B * Hq * n_splits * (mk::mla::kDv + 4) * 4;
+}
+
+int mk_attn_mla_decode_paged(const void *q, const void *cache, const int32_t *page_table,
+                             const int32_t *seq_lens, void *o, float *lse, int B, int Hq,
+                             int page_size, int max_pages, int num_pages, float scale,
+                             void *workspace, int64_t workspace_bytes, void *stream) {
+  using namespace mk;
+  if (!q || !cache || !page_table || !seq_lens || !o || !lse) return MK_ERR_INVALID_ARG;
+  if (B < 1 || Hq < 1 || max_pages < 1 || num_pages < 1) return MK_ERR_INVALID_ARG;
+  if (!std::isfinite(scale)) return MK_ERR_INVALID_ARG;
+  if (page_size != 16 && page_size != 32 && page_size != 64 && page_size != 128)
+    return MK_ERR_UNSUPPORTED;
+  if ((int64_t)num_pages * page_size > INT32_MAX || (int64_t)max_pages * page_size > INT32_MAX)
+    return MK_ERR_INVALID_ARG;
+  const int head_groups = (Hq + mla::kHeads - 1) / mla::kHeads;
+  if (B > 65535 || (int64_t)B * head_groups > 65535) return MK_ERR_UNSUPPORTED;  // grid z
+  auto misaligned = [](const void *ptr, uintptr_t a) {
+    return (reinterpret_cast<uintptr_t>(ptr) & (a - 1)) != 0;
+  };
+  if (misaligned(q, 16) || misaligned(cache, 16) || misaligned(o, 16) || misaligned(lse, 4) ||
+      misaligned(page_table, 4) || misaligned(seq_lens, 4))
+    return MK_ERR_ALIGNMENT;
+  const int sms = mla::sm_count_and_setup();
+  if (sms <= 0) return MK_ERR_CUDA;
+  const int64_t max_keys = (int64_t)max_pages * page_size;
+  const int max_blocks = (int)((max_keys + mla::kBlock - 1) / mla::kBlock);
+  mla::Params p;
+  p.page_table = page_table;
+  p.seq_lens = seq_lens;
+  p.o = reinterpret_cast<uint16_t *>(o);
+  p.lse = lse;
+  p.B = B;
+  p.Hq = Hq;
+  p.head_groups = head_groups;
+  p.page_size = page_size;
+  p.max_pages = max_pages;
+  p.num_pages = num_pages;
+  p.scale_log2 = scale * 1.4426950408889634f;
+  mla::plan(B, head_groups, max_blocks, sms, p.n_splits, p.blocks_per_split);
+  p.part = nullptr;
+  if (p.n_splits > 1) {
+    const int64_t need = (int64_t)B * Hq * p.n_splits * (mla::kDv + 4) * 4;
+    if (!workspace || workspace_bytes < need) return MK_ERR_INVALID_ARG;
+    if (misaligned(workspace, 16)) return MK_ERR_ALIGNMENT;
+    p.part = reinterpret_cast<float *>(workspace);
+  }
+  CUtensorMap tq, tc;
+  const cuuint64_t qdims[3] = {(cuuint64_t)mla::kDqk, (cuuint64_t)Hq, (cuuint64_t)B};
+  const cuuint64_t qstr[2] = {(cuuint64_t)mla::kDqk * 2, (cuuint64_t)Hq * mla::kDqk * 2};
+  const cuuint32_t qbox[3] = {(cuuint32_t)mla::kChunk, (cuuint32_t)mla::kHeads, 1};
+  const cuuint64_t cdims[2] = {(cuuint64_t)mla::kDqk, (cuuint64_t)num_pages * page_size};
+  const cuuint64_t cstr[1] = {(cuuint64_t)mla::kDqk * 2};
+  const cuuint32_t cbox[2] = {(cuuint32_t)mla::kChunk, (cuuint32_t)page_size};
+  if (!mla::encode(&tq, q, 3, qdims, qstr, qbox) || !mla::encode(&tc, cache, 2, cdims, cstr, cbox))
+    return MK_ERR_CUDA;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const dim3 grid(p.n_splits, 2, B * head_groups);
+  mla::mla_decode_kernel<<<grid, mla::kThreads, mla::kSmemBytes, st>>>(tq, tc, p);
+  if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
+  if (p.n_splits > 1) {
+    mla::mla_merge_kernel<<<(B * Hq + 3) / 4, 128, 0, st>>>(p);
+    if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
+  }
+  return MK_OK;
+}
+
+}  // extern "C"

@@ -36,14 +36,16 @@ const char *mk_attn_error_string(int status) {
 }
 
 // Synchronises the stream, then reads and clears the status words of the
-// forward, backward and decode kernels; the forward's is reported first.
+// forward, backward, decode and latent decode kernels; the first nonzero one
+// in that order is reported.
 int mk_attn_check_status(void *stream) {
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (cudaStreamSynchronize(st) != cudaSuccess) return MK_ERR_CUDA;
   const int hf = mk::fwd_take_status();
   const int hb = mk::bwd_take_status();
   const int hd = mk::decode_take_status();
-  return hf != 0 ? hf : (hb != 0 ? hb : hd);
+  const int hm = mk::mla_take_status();
+  return hf != 0 ? hf : (hb != 0 ? hb : (hd != 0 ? hd : hm));
 }
 
 int mk_attn_set_tuning(const mk_attn_tuning *t) {

@@ -50,5 +50,6 @@ mk_attn_tuning current_tuning();
 int fwd_take_status();
 int bwd_take_status();
 int decode_take_status();
+int mla_take_status();
 
 }  // namespace mk
