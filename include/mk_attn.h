@@ -290,7 +290,7 @@ MK_API int64_t mk_attn_mla_decode_workspace_bytes(int B, int Hq, int page_size, 
  *   o           bf16 [B, Hq, MK_MLA_DV] output; lse fp32 [B, Hq] output
  *               (natural log, scale included); L_b = 0 gives o = 0 and
  *               lse = -inf.
- *   Hq          any (groups of 128 heads), B * ceil(Hq / 128) <= 65535.
+ *   Hq          any (groups of 128 heads), B * ceil(Hq / 128) <= 2^29.
  *   page_size   16, 32, 64 or 128.
  *   workspace   device buffer of at least mk_attn_mla_decode_workspace_bytes()
  *               bytes, 16-byte aligned, or NULL when that is 0 (scratch for

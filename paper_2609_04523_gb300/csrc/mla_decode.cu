@@ -95,34 +95,6 @@ struct Params {
 
 __device__ __forceinline__ void record(int status) { atomicCAS(&g_status, 0, status); }
 
-// The chunks a CTA consumes, in order: for block n, the nine key chunks of
-// block n (n < nb), then the four value chunks of block n - 1 (n >= 1); the
-// value chunks of the last block close the sequence.  Step t of that order:
-// which block and which chunk (component offset / 64).
-__device__ __forceinline__ void chunk_of_step(int t, int nb, int half, int &blk, int &chunk) {
-  // Steps per block n >= 1: 9 + 4 = 13; block 0 contributes 9.
-  if (t < kChunksK) {
-    blk = 0;
-    chunk = t;
-    return;
-  }
-  const int u = t - kChunksK;
-  const int n = 1 + u / (kChunksK + kChunksV);
-  const int r = u % (kChunksK + kChunksV);
-  if (n < nb) {
-    if (r < kChunksK) {
-      blk = n;
-      chunk = r;
-    } else {
-      blk = n - 1;
-      chunk = half * kChunksV + (r - kChunksK);
-    }
-  } else {  // n == nb: the closing value chunks of block nb - 1
-    blk = nb - 1;
-    chunk = half * kChunksV + r;
-  }
-}
-
 __device__ __forceinline__ void drain_wait(uint64_t *bar, uint32_t parity) {
   int local_abort = 0;
   mbar_wait(bar, parity, &local_abort);
@@ -141,8 +113,10 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, u
 __global__ void __launch_bounds__(kThreads, 1)
     mla_decode_kernel(const __grid_constant__ CUtensorMap tm_q,
                       const __grid_constant__ CUtensorMap tm_c, const Params p) {
-  const int split = blockIdx.x, half = blockIdx.y;
-  const int b = blockIdx.z / p.head_groups, hg = blockIdx.z % p.head_groups;
+  // blockIdx.x = 2 (b * head_groups + hg) + half, blockIdx.y = split: every
+  // sequence's first (largest) split is dispatched before any second one.
+  const int split = blockIdx.y, half = blockIdx.x & 1;
+  const int b = (blockIdx.x >> 1) / p.head_groups, hg = (blockIdx.x >> 1) % p.head_groups;
   const int PS = p.page_size;
   int L = p.seq_lens[b];
   if (L < 0 || L > p.max_pages * PS) {
@@ -186,7 +160,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after_sync();
   const uint32_t tmem = ctl->tmem_base;
   volatile int *abort = &ctl->abort;
-  const int n_steps = nb == 0 ? 0 : kChunksK + (nb - 1) * (kChunksK + kChunksV) + kChunksV;
+  // Chunks a CTA consumes, in order: the nine key chunks of block n, then
+  // the four value chunks of block n - 1 (the MMAs' order), 13 per block.
+  const int n_steps = nb * (kChunksK + kChunksV);
 
   if (warp == kLoadWarp) {
     // ------------------------------------------------------------ producer
@@ -205,32 +181,58 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
     }
     const uint64_t pol_c = l2_policy_evict_last();  // read again for the values
-    const int pages_per_block = kBlock / PS;
-    for (int t = 0; ok && t < n_steps; ++t) {
-      const int s = t % kSlots;
-      ok = mbar_wait_all(&ctl->slot_empty[s], ((t / kSlots) & 1) ^ 1, abort);
-      if (!ok) break;
-      if (elect_one()) {
-        int blk, chunk;
-        chunk_of_step(t, nb, half, blk, chunk);
-        const int page0 = (first + blk) * pages_per_block;  // logical page of the block's row 0
-        const int n_pages_seq = (L + PS - 1) / PS;
-        mbar_arrive_expect_tx(&ctl->slot_full[s], kChunkBytes);
-        uint8_t *dst = smem + kOffRing + s * kChunkBytes;
-        for (int i = 0; i < pages_per_block; ++i) {
-          // Pages past the sequence end load its first page of the block
-          // instead (finite rows, masked out), so the byte count holds.
-          const int lp = page0 + i < n_pages_seq ? page0 + i : page0;
-          int page = p.page_table[(int64_t)b * p.max_pages + lp];
-          if (page < 0 || page >= p.num_pages) {
-            record(MK_ERR_INVALID_ARG);
-            page = 0;
-          }
-          tma_load_2d(dst + i * PS * 128, &tm_c, &ctl->slot_full[s], chunk * kChunk, page * PS,
-                      pol_c);
+    const int pages_per_block = kBlock / PS;  // 1..8
+    const int n_pages_seq = (L + PS - 1) / PS;
+    const int lane = lane_id();
+    // Physical page of page `lane` of block n (lanes < pages_per_block), one
+    // global load per lane per block, loaded one block ahead.  Pages past the
+    // sequence end take the block's first page instead (finite rows, masked
+    // out), so every chunk moves the same number of bytes.
+    auto block_pages = [&](int n) {
+      int page = 0;
+      if (n < nb && lane < pages_per_block) {
+        const int page0 = (first + n) * pages_per_block;
+        const int lp = page0 + lane < n_pages_seq ? page0 + lane : page0;
+        page = p.page_table[(int64_t)b * p.max_pages + lp];
+        if (page < 0 || page >= p.num_pages) {
+          record(MK_ERR_INVALID_ARG);
+          page = 0;
         }
       }
+      return page;
+    };
+    int t = 0;  // chunk step: the same order the MMA warp consumes
+    // One chunk (128 keys x 64 components at component offset 64 * chunk) of
+    // the block whose pages are in `pages` (lane i: page i).
+    auto load_chunk = [&](int pages, int chunk) {
+      const int s = t % kSlots;
+      ok = mbar_wait_all(&ctl->slot_empty[s], ((t / kSlots) & 1) ^ 1, abort);
+      if (!ok) return;
+      int pg[kBlock / 16];
+#pragma unroll
+      for (int i = 0; i < kBlock / 16; ++i) pg[i] = __shfl_sync(0xffffffffu, pages, i);
+      if (elect_one()) {
+        mbar_arrive_expect_tx(&ctl->slot_full[s], kChunkBytes);
+        uint8_t *dst = smem + kOffRing + s * kChunkBytes;
+#pragma unroll
+        for (int i = 0; i < kBlock / 16; ++i)
+          if (i < pages_per_block)
+            tma_load_2d(dst + i * PS * 128, &tm_c, &ctl->slot_full[s], chunk * kChunk, pg[i] * PS,
+                        pol_c);
+      }
       __syncwarp();
+      ++t;
+    };
+    int pages_prev = 0, pages_cur = block_pages(0);
+    for (int n = 0; ok && n <= nb; ++n) {
+      const int pages_next = block_pages(n + 1);
+      // The nine key chunks of block n, then the value chunks of block n-1.
+      if (n < nb)
+        for (int c = 0; ok && c < kChunksK; ++c) load_chunk(pages_cur, c);
+      if (n >= 1)
+        for (int c = 0; ok && c < kChunksV; ++c) load_chunk(pages_prev, half * kChunksV + c);
+      pages_prev = pages_cur;
+      pages_cur = pages_next;
     }
     // Teardown: the loads issued land before the CTA exits.
     if (nb > 0) drain_wait(&ctl->q_full, 0);
@@ -583,7 +585,7 @@ int mk_attn_mla_decode_paged(const void *q, const void *cache, const int32_t *pa
   if ((int64_t)num_pages * page_size > INT32_MAX || (int64_t)max_pages * page_size > INT32_MAX)
     return MK_ERR_INVALID_ARG;
   const int head_groups = (Hq + mla::kHeads - 1) / mla::kHeads;
-  if (B > 65535 || (int64_t)B * head_groups > 65535) return MK_ERR_UNSUPPORTED;  // grid z
+  if ((int64_t)B * head_groups > (1 << 29)) return MK_ERR_UNSUPPORTED;  // grid x
   auto misaligned = [](const void *ptr, uintptr_t a) {
     return (reinterpret_cast<uintptr_t>(ptr) & (a - 1)) != 0;
   };
@@ -624,7 +626,7 @@ int mk_attn_mla_decode_paged(const void *q, const void *cache, const int32_t *pa
   if (!mla::encode(&tq, q, 3, qdims, qstr, qbox) || !mla::encode(&tc, cache, 2, cdims, cstr, cbox))
     return MK_ERR_CUDA;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  const dim3 grid(p.n_splits, 2, B * head_groups);
+  const dim3 grid(2 * B * head_groups, p.n_splits, 1);
   mla::mla_decode_kernel<<<grid, mla::kThreads, mla::kSmemBytes, st>>>(tq, tc, p);
   if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
   if (p.n_splits > 1) {
