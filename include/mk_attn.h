@@ -331,6 +331,8 @@ typedef struct {
   int split_ctas_per_sm; /* decode: KV splits are planned for about this many
                             CTAs per SM, 1..64 (default 24) */
   int split_min_pages;   /* decode: fewest pages per KV split, 1..4096 (default 2) */
+  int mla_split_ctas_per_sm; /* latent decode: KV splits planned for about this many
+                                CTAs per SM (one CTA fits an SM), 1..64 (default 3) */
 } mk_attn_tuning;
 
 /*

@@ -35,6 +35,7 @@ SPACES = {
                      schedule=[binding.SCHED_SNAKE, binding.SCHED_ROUND_ROBIN,
                                binding.SCHED_BLOCKED]),
     "decode": dict(split_ctas_per_sm=[3, 6, 12, 24, 48], split_min_pages=[1, 2, 4, 8, 16]),
+    "mla": dict(mla_split_ctas_per_sm=[1, 2, 3, 4, 6, 8, 12, 16, 24]),
 }
 
 
@@ -67,6 +68,14 @@ def make_step(workload: str, config: int, dev):
     inputs and its work per call (FLOPs, or bytes for decode)."""
     import numpy as np
     import torch
+    if workload == "mla":
+        lens = [int(x) for x in np.random.default_rng(2001).integers(1024, 8193, size=64)]
+        inp = W.make_mla_paged(lens, 128, 64, seed=2002, spare_pages=64)
+        args = [t.to(dev) for t in (inp.q, inp.cache, inp.page_table, inp.seq_lens)]
+
+        def step():  # the workspace follows the current split plan
+            binding.mla_decode_paged(*args, scale=inp.scale)
+        return step, W.mla_decode_bytes(lens, 128), "GB/s"
     if workload == "decode":
         lens = [int(x) for x in np.random.default_rng(2001).integers(1024, 8193, size=64)]
         inp = W.make_paged(lens, 32, 8, 128, 64, seed=2001, spare_pages=64)

@@ -35,14 +35,14 @@ class MkAttnTuning(ctypes.Structure):
     """mk_attn_tuning: launch parameters that change speed, not results."""
     _fields_ = [("ctas", ctypes.c_int), ("schedule", ctypes.c_int),
                 ("rescale_log2", ctypes.c_float), ("split_ctas_per_sm", ctypes.c_int),
-                ("split_min_pages", ctypes.c_int)]
+                ("split_min_pages", ctypes.c_int), ("mla_split_ctas_per_sm", ctypes.c_int)]
 
     def as_dict(self) -> dict:
         return {name: getattr(self, name) for name, _ in self._fields_}
 
 
 DEFAULT_TUNING = dict(ctas=0, schedule=SCHED_SNAKE, rescale_log2=8.0, split_ctas_per_sm=24,
-                      split_min_pages=2)
+                      split_min_pages=2, mla_split_ctas_per_sm=3)
 
 # Bytes of the library's own decode scratch array (MK_ATTN_DECODE_STATIC_SCRATCH_BYTES).
 DECODE_STATIC_SCRATCH_BYTES = 16 * 1024 * 1024

@@ -67,7 +67,6 @@ constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColS = 0;      // S buffer X at kColS + 128 X
 constexpr uint32_t kColO = 256;    // O: 256 columns
 constexpr float kRescaleThreshold = 8.0f;
-constexpr int kSplitCtasPerSm = 2;  // split planning: about two waves of CTAs
 
 __device__ int g_status = 0;
 
@@ -523,11 +522,13 @@ static int sm_count_and_setup() {
   return di.attr == cudaSuccess ? di.sm_count : 0;
 }
 
-// KV splits of whole 128-key blocks: about kSplitCtasPerSm CTAs per SM over
-// B x head groups x 2 value halves.
+// KV splits of whole 128-key blocks: about mla_split_ctas_per_sm (process-wide
+// tuning) CTAs per SM over B x head groups x 2 value halves.  One CTA fills
+// an SM, so this is the number of waves: more, shorter splits even out
+// unequal sequence lengths, at the cost of a Q load and a merge row each.
 static void plan(int B, int head_groups, int max_blocks, int sms, int &n_splits, int &bps) {
   const int64_t units = (int64_t)B * head_groups * 2;
-  int64_t want = ((int64_t)kSplitCtasPerSm * sms + units - 1) / units;
+  int64_t want = ((int64_t)current_tuning().mla_split_ctas_per_sm * sms + units - 1) / units;
   want = want < 1 ? 1 : (want > max_blocks ? max_blocks : want);
   bps = (int)((max_blocks + want - 1) / want);
   n_splits = (max_blocks + bps - 1) / bps;

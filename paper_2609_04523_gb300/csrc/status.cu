@@ -9,7 +9,7 @@
 
 namespace mk {
 namespace {
-constexpr mk_attn_tuning kDefaultTuning = {0, MK_SCHED_SNAKE, 8.0f, 24, 2};
+constexpr mk_attn_tuning kDefaultTuning = {0, MK_SCHED_SNAKE, 8.0f, 24, 2, 3};
 std::mutex g_tuning_mu;
 mk_attn_tuning g_tuning = kDefaultTuning;
 }  // namespace
@@ -56,6 +56,7 @@ int mk_attn_set_tuning(const mk_attn_tuning *t) {
     if (!(t->rescale_log2 >= 0.0f && t->rescale_log2 <= 16.0f)) return MK_ERR_INVALID_ARG;
     if (t->split_ctas_per_sm < 1 || t->split_ctas_per_sm > 64) return MK_ERR_INVALID_ARG;
     if (t->split_min_pages < 1 || t->split_min_pages > 4096) return MK_ERR_INVALID_ARG;
+    if (t->mla_split_ctas_per_sm < 1 || t->mla_split_ctas_per_sm > 64) return MK_ERR_INVALID_ARG;
     v = *t;
   }
   std::lock_guard<std::mutex> lock(mk::g_tuning_mu);

@@ -22,7 +22,7 @@ def test_defaults():
     ("ctas", -1), ("ctas", 65536), ("schedule", -1), ("schedule", 3),
     ("rescale_log2", -0.5), ("rescale_log2", 16.5), ("rescale_log2", float("nan")),
     ("split_ctas_per_sm", 0), ("split_ctas_per_sm", 65), ("split_min_pages", 0),
-    ("split_min_pages", 4097)])
+    ("split_min_pages", 4097), ("mla_split_ctas_per_sm", 0), ("mla_split_ctas_per_sm", 65)])
 def test_out_of_range_is_rejected_and_changes_nothing(field, bad):
     binding.set_tuning(ctas=77)
     t = binding.MkAttnTuning(**{**binding.DEFAULT_TUNING, field: bad})

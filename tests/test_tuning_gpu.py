@@ -119,6 +119,25 @@ def test_decode_split_plans(plan):
     assert float(np.max(np.abs(lse[live] - lse_ref[live]))) <= 1e-3
 
 
+@pytest.mark.parametrize("waves", [1, 24])
+def test_mla_split_plans(waves):
+    """The latent decode step under one and many KV splits: parity."""
+    inp = W.make_mla_paged([3000, 1, 0, 700], 64, 64, seed=955)
+    dev = torch.device("cuda")
+    args = [t.to(dev) for t in (inp.q, inp.cache, inp.page_table, inp.seq_lens)]
+    with binding.tuning(mla_split_ctas_per_sm=waves):
+        o, lse = binding.mla_decode_paged(*args, scale=inp.scale)
+        assert binding.mk_attn_check_status(torch.cuda.current_stream().cuda_stream) == 0
+    o_ref, lse_ref = oracle.mla_decode(inp.q, inp.cache, inp.page_table, inp.seq_lens, inp.scale,
+                                       inp.dv)
+    o, lse = o.float().cpu().numpy(), lse.double().cpu().numpy()
+    live = np.asarray(inp.seq_lens) > 0
+    assert np.all(o[~live] == 0) and np.all(np.isneginf(lse[~live]))
+    d = o[live] - o_ref[live]
+    assert float(np.max(np.abs(d))) <= 2e-2
+    assert float(np.max(np.abs(lse[live] - lse_ref[live]))) <= 1e-3
+
+
 def test_sweep_returns_sorted_rows_and_restores_tuning():
     binding.set_tuning(ctas=99)
     rows = autotune.sweep("prefill", 1, space={"ctas": [0, 2], "schedule": [0, 2]}, steps=2,
