@@ -121,3 +121,33 @@ def test_bwd_causal_gqa_b4_s2048():
     inp = W.make_config_inputs(2)
     do = W.make_grad_out(inp.q.shape, seed=inp.cfg.seed)
     check(inp.q, inp.k, inp.v, do, True, inp.cfg.scale, what="B4 S2048")
+
+
+def test_bwd_causal_gqa_b1_s32768_sampled():
+    """The long-context workload (causal GQA B=1, Hq=32, Hkv=8, S=32768,
+    D=128, N(0, 0.5^2)) at full size: dq on sampled rows (a row's dq depends on
+    that row only), dk / dv on the last key tile of every key/value head and on
+    a range further back (the oracle visits every query row that sees them),
+    and two identities over the whole tensors: sum_j dk_j = 0 (the rows of dS
+    sum to zero) and sum_j dv_j = sum over the group's heads of sum_i dO_i."""
+    inp = W.make_config_inputs(3)
+    c = inp.cfg
+    do = W.make_grad_out(inp.q.shape, seed=c.seed)
+    dq, dk, dv = gpu_fwd_bwd(inp.q, inp.k, inp.v, do, True, c.scale)
+    S, G = c.S, c.Hq // c.Hkv
+    rows = [(0, h, i) for h in (0, 13, 31) for i in (0, 1, 127, 128, 4097, 20000, S - 129, S - 1)]
+    ref = oracle.attn_bwd_dq_rows(inp.q, inp.k, inp.v, do, True, c.scale, rows)
+    compare(np.stack([dq[0, i, h] for _, h, i in rows]), ref, "sampled dq rows")
+    ranges = [(0, g, S - 128, S) for g in range(c.Hkv)] + [(0, 5, S - 1024, S - 1016)]
+    rk, rv = oracle.attn_bwd_dkv_ranges(inp.q, inp.k, inp.v, do, True, c.scale, ranges)
+    gk = np.concatenate([dk[0, j0:j1, g] for _, g, j0, j1 in ranges])
+    gv = np.concatenate([dv[0, j0:j1, g] for _, g, j0, j1 in ranges])
+    compare(gk, rk, "sampled dk ranges")
+    compare(gv, rv, "sampled dv ranges")
+    dof = do.double().numpy()[0]
+    for g in range(c.Hkv):
+        sk = dk[0, :, g].astype(np.float64).sum(axis=0)
+        assert np.max(np.abs(sk)) <= 1e-2 * np.max(np.abs(dk[0, :, g])) * math.sqrt(S), "sum of dk"
+        want = dof[:, g * G:(g + 1) * G].sum(axis=(0, 1))
+        sv = dv[0, :, g].astype(np.float64).sum(axis=0)
+        assert np.max(np.abs(sv - want)) <= 1e-2 * np.max(np.abs(want)), "sum of dv"

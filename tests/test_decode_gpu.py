@@ -158,3 +158,12 @@ def test_decode_device_side_range_errors_are_reported():
     binding.decode_paged(*args, scale=bad.scale)
     assert binding.mk_attn_check_status(st) == binding.MK_ERR_INVALID_ARG
     check(inp, "after range errors")
+
+
+def test_decode_bench_workload():
+    """The bench workload (64 sequences of 1024-8192 cached tokens, Hq 32,
+    Hkv 8, D 128, page 64, pages in random order), every output row against
+    the oracle, in the launch configuration bench.py times."""
+    lens = [int(x) for x in np.random.default_rng(2001).integers(1024, 8193, size=64)]
+    inp = W.make_paged(lens, 32, 8, 128, 64, seed=2001, spare_pages=64)
+    check(inp, "bench workload")

@@ -85,3 +85,12 @@ def test_mla_rejects_bad_arguments():
                      (dict(scale=float("inf")), binding.MK_ERR_INVALID_ARG)):
         assert binding.mk_attn_mla_decode_paged(**{**good, **kw}) == want, kw
     del dev
+
+
+def test_mla_bench_workload():
+    """The bench workload (64 sequences of 1024-8192 cached tokens, 128 heads,
+    page 64, pages in random order), every output row against the oracle, in
+    the launch configuration bench.py times."""
+    lens = [int(x) for x in np.random.default_rng(2001).integers(1024, 8193, size=64)]
+    inp = W.make_mla_paged(lens, 128, 64, seed=2002, spare_pages=64)
+    check(inp, "bench workload")
