@@ -412,6 +412,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t pol_q = l2_policy_evict_first();
       const uint64_t pol_kv = l2_policy_evict_last();
       uint32_t q_iter = 0, it = 0, n_pub = 0;
+      uint32_t q_issued[2] = {0, 0};  // Q loads issued per tile, for the teardown drain
       auto publish = [&](const Unit &w) {
         const int e = n_pub % kUnitRing;
         if (elect_one()) {
@@ -433,9 +434,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (p.stall_first_slot) break;
         const int hkv = w.hq / p.group;
         const int n_blk = max(tile_blocks(p, w, 0), tile_blocks(p, w, 1));
-        for (int x = 0; x < 2; ++x) {
+        // Q_A, then K_0, then Q_B: the unit's first S (tile A) needs only the
+        // first two, so it starts a tile-load earlier.
+        auto load_q = [&](int x) {
           ok = mbar_wait_all(&ctl->bar_q_empty[x], (q_iter & 1) ^ 1, abort);
-          if (!ok) break;
+          if (!ok) return;
           if (elect_one()) {
             mbar_arrive_expect_tx(&ctl->bar_q_full[x], C::kTileBytes);
 #pragma unroll
@@ -445,9 +448,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                           w.seq_start + (2 * w.pair + x) * kTile, pol_q);
           }
           __syncwarp();
-        }
+          ++q_issued[x];
+        };
+        load_q(0);
         if (!ok) break;
-        ++q_iter;
         for (int j = 0; j <= n_blk; ++j) {
           const int s = it % NS;
           ok = mbar_wait_all(&ctl->bar_kv_empty[s], ((it / NS) & 1) ^ 1, abort);
@@ -472,6 +476,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           __syncwarp();
           ++it;
+          if (j == 0) {
+            load_q(1);
+            if (!ok) break;
+            ++q_iter;
+          }
         }
       }
       {
@@ -480,8 +489,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // Teardown: every load issued must land before the CTA exits.  For each
       // slot the last issued phase is waited for (earlier phases precede it).
-      if (q_iter > 0)
-        for (int x = 0; x < 2; ++x) drain_wait(&ctl->bar_q_full[x], (q_iter - 1) & 1);
+      for (int x = 0; x < 2; ++x)
+        if (q_issued[x] > 0) drain_wait(&ctl->bar_q_full[x], (q_issued[x] - 1) & 1);
       for (uint32_t n = (it > (uint32_t)NS ? it - NS : 0); n < it; ++n)
         drain_wait(&ctl->bar_kv_full[n % NS], (n / NS) & 1);
     } else if (warp == kMmaWarp) {
@@ -536,8 +545,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!w.valid) break;
         const int nx[2] = {tile_blocks(p, w, 0), tile_blocks(p, w, 1)};
         const int n_blk = max(nx[0], nx[1]);
-        for (int x = 0; x < 2 && ok; ++x)
-          ok = mbar_wait_all(&ctl->bar_q_full[x], q_iter & 1, abort);
         const int n_min = min(nx[0], nx[1]);
         // Generic iteration j: any mix of P V and S per tile (unit edges).
         auto edge_iteration = [&](int j) {
@@ -546,6 +553,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int x = 0; x < 2; ++x) {
             if (!ok) break;
+            // Iteration 0 waits for Q_X (loaded after K_0 for tile B), also
+            // when the tile has no key block: its Q_empty commit below must
+            // not release a load still in flight.
+            if (j == 0) {
+              ok = mbar_wait_all(&ctl->bar_q_full[x], q_iter & 1, abort);
+              if (!ok) break;
+            }
             const bool do_pv = j > 0 && j - 1 < nx[x];
             const bool do_s = j < nx[x];
             if (do_pv) {
