@@ -129,8 +129,9 @@ MK_API int64_t mk_attn_bwd_workspace_bytes(int B, int Hq, int S, int varlen);
  *   workspace  device buffer of at least mk_attn_bwd_workspace_bytes()
  *              bytes, 16-byte aligned; scratch, contents on entry do not
  *              matter.  Calls that share a workspace must not overlap.
- *   stream     cudaStream_t; three kernels are enqueued (Delta, dK/dV, dQ),
- *              the call never synchronises.
+ *   stream     cudaStream_t; two kernels are enqueued (dQ, which also
+ *              writes Delta_i = dO_i . o_i to the workspace, then dK/dV,
+ *              which reads it); the call never synchronises.
  * Layout and alignment: as mk_attn_fwd; dO, dq, dk, dv and workspace 16-byte
  * aligned, lse 4-byte aligned.
  * Returns MK_OK, or MK_ERR_INVALID_ARG (null pointer, sizes, too small a
@@ -147,19 +148,19 @@ MK_API int mk_attn_bwd(const void *q, const void *k, const void *v, const void *
                        void *stream);
 
 /* Stages of the backward pass, for mk_attn_bwd_stages. */
-#define MK_BWD_DELTA 1 /* Delta_i = dO_i . o_i into the workspace */
+#define MK_BWD_DELTA 1 /* Delta_i = dO_i . o_i into the workspace (a kernel of its own) */
 #define MK_BWD_DKDV 2  /* dk and dv (reads Delta from the workspace) */
-#define MK_BWD_DQ 4    /* dq (reads Delta from the workspace) */
+#define MK_BWD_DQ 4    /* dq; also computes Delta and writes it to the workspace */
 #define MK_BWD_ALL 7
 
 /*
  * mk_attn_bwd_stages -- mk_attn_bwd, enqueuing only the stages in `stages`
- * (a nonzero OR of the MK_BWD_* flags), in the order Delta, dK/dV, dQ.
- * Arguments, checks and errors are those of mk_attn_bwd.  MK_BWD_DKDV and
- * MK_BWD_DQ read the Delta that an earlier MK_BWD_DELTA stage wrote into the
- * same workspace for the same o and dO; once it is there, the two are
- * independent of each other (e.g. on two streams, ordered after Delta by the
- * caller).  Outputs of stages not enqueued are left untouched.
+ * (a nonzero OR of the MK_BWD_* flags), in the order Delta, dQ, dK/dV; the
+ * Delta kernel is skipped when dQ is enqueued (dQ writes Delta itself).
+ * Arguments, checks and errors are those of mk_attn_bwd.  MK_BWD_DKDV reads
+ * the Delta that an earlier MK_BWD_DELTA or MK_BWD_DQ stage wrote into the
+ * same workspace for the same o and dO.  Outputs of stages not enqueued are
+ * left untouched.
  */
 MK_API int mk_attn_bwd_stages(const void *q, const void *k, const void *v, const void *o,
                               const float *lse, const void *dO, void *dq, void *dk, void *dv,

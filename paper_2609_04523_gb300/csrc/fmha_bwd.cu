@@ -11,8 +11,10 @@
 //   dq_i    = scale * sum_j dS_ij k_j
 //   dk_j    = scale * sum_{h in group} sum_i dS_ij q_i
 //
-// Three kernels, all deterministic (no atomics):
-//   delta_kernel   Delta_i = dO_i . o_i from the forward's bf16 o (fp32).
+// Kernels, all deterministic (no atomics), launched dQ first:
+//   delta_kernel   Delta_i = dO_i . o_i from the forward's bf16 o (fp32); only
+//                  for callers that want Delta without dQ (the dQ kernel
+//                  computes it for its own rows and stores it).
 //   bwd_kernel<D, false> (dK/dV): a unit is (sequence, key/value head g,
 //                  128-key tile); it holds K and V and streams the Q and dO
 //                  tiles of every query head of g's group (causal: the query
@@ -20,8 +22,10 @@
 //                  dP^T = V dO^T in TMEM (lanes = keys), P^T and dS^T written
 //                  back to TMEM as bf16, dV += P^T dO and dK += dS^T Q.
 //   bwd_kernel<D, true> (dQ): a unit is (sequence, query head, 128-row query
-//                  tile); it holds Q and dO and streams K and V tiles, with
-//                  S = Q K^T, dP = dO V^T, dS to TMEM and dQ += dS K.
+//                  tile); it holds Q and dO (and computes the tile's Delta
+//                  from dO and o, writing it for the dK/dV kernel), streams K
+//                  and V tiles, with S = Q K^T, dP = dO V^T, dS to TMEM and
+//                  dQ += dS K.
 // dQ recomputes S and dP instead of accumulating partial dQ tiles across
 // CTAs, which keeps the result deterministic and needs no fp32 scratch.
 //
@@ -100,8 +104,9 @@ struct Cfg {
   static constexpr int kOffX2 = kTileBytes;      // V (dK/dV) or dO (dQ)
   static constexpr int kOffY1 = 2 * kTileBytes;  // Y1 ring: Q (dK/dV) or K (dQ)
   static constexpr int kOffY2 = kOffY1 + kStages1 * kTileBytes;  // Y2 ring: dO or V
-  static constexpr int kOffVec = kOffY2 + kStages2 * kTileBytes;  // dK/dV: [stage][lse2 | delta][128]
-  static constexpr int kOffCtl = kOffVec + (DQ ? 0 : kStages1 * 2 * kTile * 4);
+  // dK/dV: [stage][lse2 | delta][128]; dQ: [warpgroup][128] halves of Delta
+  static constexpr int kOffVec = kOffY2 + kStages2 * kTileBytes;
+  static constexpr int kOffCtl = kOffVec + (DQ ? 2 * kTile * 4 : kStages1 * 2 * kTile * 4);
   static constexpr int kSmemBytes = kOffCtl + 256 + 1024;
   static_assert(kSmemBytes <= 232448, "shared memory per CTA");
 };
@@ -114,6 +119,7 @@ struct Ctl {
   uint64_t fixed_full, fixed_empty;
   uint64_t y1_full[4], y1_empty[4], y2_full[4], y2_empty[4];
   uint64_t s_full, dp_full, p_full, dp_free, ds_full, acc_full, mma_drained;
+  uint64_t dx_full;  // dQ: both warpgroups' halves of the unit's Delta are in shared memory
   uint32_t tmem_base;
   int abort;
 };
@@ -121,7 +127,8 @@ static_assert(sizeof(Ctl) <= 256, "control block");
 
 struct Params {
   const float *lse;          // [B, Hq, S] or [Hq, T]
-  const float *delta;        // same layout
+  float *delta;              // same layout: written by the dQ kernel, read by dK/dV
+  const uint16_t *o;         // bf16, layout of q (the dQ kernel's Delta)
   uint16_t *dq, *dk, *dv;    // bf16, layouts of q, k, v
   const int32_t *cu_seqlens;
   int B, Hq, Hkv, S, G;      // S: tokens per sequence, or total tokens T (varlen)
@@ -227,6 +234,10 @@ __device__ __forceinline__ int unit_of_round(int k, int schedule, int n_units) {
   return (k & 1) ? (k + 1) * G - 1 - c : k * G + c;
 }
 
+__device__ __forceinline__ void prefetch_l2(const void *ptr) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(ptr));
+}
+
 __device__ __forceinline__ void drain_wait(uint64_t *bar, uint32_t parity) {
   int local_abort = 0;
   mbar_wait(bar, parity, &local_abort);
@@ -255,7 +266,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(&ctl->fixed_full, 1);
-    mbar_init(&ctl->fixed_empty, 1);
+    // dQ: the fixed tiles are free once the MMAs are done with them and the
+    // elementwise warps have read the dO tile for Delta.
+    mbar_init(&ctl->fixed_empty, DQ ? 2 : 1);
     for (int s = 0; s < NS1; ++s) {
       // Y1 of dK/dV: the TMA bytes plus one arrival per producer lane for
       // the lse / Delta vectors the lanes write.
@@ -273,6 +286,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&ctl->ds_full, kEwThreads);
     mbar_init(&ctl->acc_full, 1);
     mbar_init(&ctl->mma_drained, 1);
+    mbar_init(&ctl->dx_full, kEwThreads);
     ctl->abort = 0;
     fence_mbar_init();
   }
@@ -548,18 +562,39 @@ __global__ void __launch_bounds__(kThreads, 1)
       int first_q = 0;
       const int N = unit_iters<DQ>(p, w, first_q);
       const int nq = tiles_of(w.len) - first_q;
-      // dQ: this thread's query row, its lse (base 2) and Delta.
+      // dQ: this thread's query row, its lse (base 2) and Delta = dO . o.
+      // The lse and this warpgroup's half of the o row are loaded here (the
+      // previous unit prefetched them into L2) and used in the first key
+      // tile: lse for P, and o, with the dO tile in shared memory, for Delta,
+      // which the first dS needs and the dK/dV kernel reads back.
       const int qpos = w.tile * kTile + row;
-      float row_l2 = INFINITY, row_dl = 0.f;
+      float row_l2 = INFINITY, row_dl = 0.f, lse_raw = INFINITY;
+      int64_t ri = 0;
+      uint4 ov[DQ ? D / 16 : 1];
       if constexpr (DQ) {
         if (qpos < w.len) {
-          const int64_t ri = row_index(p, w, w.head, qpos);
-          row_l2 = p.lse[ri] * kLog2e;
-          row_dl = p.delta[ri];
+          ri = row_index(p, w, w.head, qpos);
+          lse_raw = p.lse[ri];
+          const uint16_t *orow = p.o + (((int64_t)w.seq_start + qpos) * p.Hq + w.head) * D + wg * (D / 2);
+#pragma unroll
+          for (int c8 = 0; c8 < D / 16; ++c8) ov[c8] = *reinterpret_cast<const uint4 *>(orow + c8 * 8);
         }
       }
       for (int n = 0; n < N; ++n) {
         const uint32_t i = it + n;
+        if constexpr (DQ) {
+          if (n == N - 1) {  // last key tile: bring the next unit's o and lse rows into L2
+            const int un = unit_of_round(k + 1, p.schedule, p.n_units);
+            if (un < p.n_units) {
+              const Unit wn = map_unit<DQ>(p, un);
+              const int qn = wn.tile * kTile + row;
+              if (wn.valid && qn < wn.len) {
+                prefetch_l2(p.o + (((int64_t)wn.seq_start + qn) * p.Hq + wn.head) * D + wg * (D / 2));
+                if (wg == 0) prefetch_l2(p.lse + row_index(p, wn, wn.head, qn));
+              }
+            }
+          }
+        }
         ok = mbar_wait_all(&ctl->s_full, n_s & 1, abort);
         if (!ok) break;
         tc_fence_after_sync();
@@ -580,6 +615,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           // S(n) is in registers: S(n+1) may overwrite it.
           tc_fence_before_sync();
           mbar_arrive(&ctl->p_full);
+          if (n == 0) row_l2 = lse_raw * kLog2e;
           const int kpos0 = n * kTile + col0;  // key position of column 0 of this half
           const int lim = p.causal ? min(w.len, qpos + 1) : w.len;  // keys [0, lim)
           const bool mask = kpos0 + 64 > lim;
@@ -587,6 +623,41 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int c = 0; c < 64; ++c) {
             const float e = ex2_approx(fmaf(x[c], c2, -row_l2));
             x[c] = (!mask || kpos0 + c < lim) ? e : 0.f;
+          }
+          if (n == 0) {
+            ok = mbar_wait_all(&ctl->fixed_full, (n_unit & 1), abort);  // the dO tile has landed
+            if (!ok) break;
+            float part = 0.f;
+            if (qpos < w.len) {
+              const uint8_t *dorow = smem + C::kOffX2;
+#pragma unroll
+              for (int c8 = 0; c8 < D / 16; ++c8) {  // this warpgroup's D/2 components, 8 at a time
+                const int e0 = wg * (D / 2) + c8 * 8;
+                const int chunk = (e0 % kBoxCols) / 8;
+                const uint4 dv4 = *reinterpret_cast<const uint4 *>(
+                    dorow + (e0 / kBoxCols) * kBoxBytes + row * 128 + ((chunk ^ (row & 7)) << 4));
+                const uint32_t aw[4] = {dv4.x, dv4.y, dv4.z, dv4.w};
+                const uint32_t bw[4] = {ov[c8].x, ov[c8].y, ov[c8].z, ov[c8].w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                  part = fmaf(__uint_as_float(aw[e] << 16), __uint_as_float(bw[e] << 16), part);
+                  part = fmaf(__uint_as_float(aw[e] & 0xffff0000u), __uint_as_float(bw[e] & 0xffff0000u), part);
+                }
+              }
+            }
+            // The two warpgroups' halves meet in vec.  A warpgroup writes the
+            // next unit's half only after this unit's dQ accumulation, which
+            // needs both warpgroups' first dS: no overwrite.  The exchange is
+            // an mbarrier with a bounded wait, so a warpgroup that unwinds on
+            // a timeout cannot leave the other one waiting for ever.
+            vec[wg * kTile + row] = part;
+            mbar_arrive(&ctl->dx_full);
+            ok = mbar_wait_all(&ctl->dx_full, n_unit & 1, abort);
+            if (!ok) break;
+            // Every elementwise thread has read the dO tile: release it.
+            if (threadIdx.x == 0) mbar_arrive(&ctl->fixed_empty);
+            row_dl = vec[row] + vec[kTile + row];
+            if (wg == 0 && qpos < w.len) p.delta[ri] = row_dl;
           }
         } else {
           // The producer lanes wrote this slot's vectors before arriving on
@@ -790,7 +861,9 @@ static int launch(const void *q, const void *k, const void *v, const void *o, co
   const int v0 = D == 128 ? 2 : 0;
   if (di.sm_count <= 0 || di.attr_err[v0] != cudaSuccess || di.attr_err[v0 + 1] != cudaSuccess)
     return MK_ERR_CUDA;
-  if (stages & 1) {
+  // The dQ kernel computes Delta for its own rows; the separate Delta kernel
+  // runs only when Delta is asked for without dQ.
+  if ((stages & MK_BWD_DELTA) && !(stages & MK_BWD_DQ)) {
     const dim3 grid((unsigned)((tokens + 15) / 16), (unsigned)p.Hq);
     delta_kernel<D><<<grid, 256, 0, st>>>(
         reinterpret_cast<const uint16_t *>(o), reinterpret_cast<const uint16_t *>(dO),
@@ -806,14 +879,14 @@ static int launch(const void *q, const void *k, const void *v, const void *o, co
   Params pk = p, pq = p;
   pk.n_units = (int)(tiles * p.Hkv);
   pq.n_units = (int)(tiles * p.Hq);
-  if (stages & 2) {
-    const int gk = pk.n_units < ctas ? pk.n_units : ctas;
-    bwd_kernel<D, false><<<gk, kThreads, Cfg<D, false>::kSmemBytes, st>>>(tq, tk, tv, tdo, pk);
-    if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
-  }
-  if (stages & 4) {
+  if (stages & MK_BWD_DQ) {
     const int gq = pq.n_units < ctas ? pq.n_units : ctas;
     bwd_kernel<D, true><<<gq, kThreads, Cfg<D, true>::kSmemBytes, st>>>(tq, tk, tv, tdo, pq);
+    if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
+  }
+  if (stages & MK_BWD_DKDV) {
+    const int gk = pk.n_units < ctas ? pk.n_units : ctas;
+    bwd_kernel<D, false><<<gk, kThreads, Cfg<D, false>::kSmemBytes, st>>>(tq, tk, tv, tdo, pk);
     if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
   }
   return MK_OK;
@@ -871,7 +944,8 @@ int mk_attn_bwd_stages(const void *q, const void *k, const void *v, const void *
   if (tiles * Hq > INT32_MAX) return MK_ERR_INVALID_ARG;
   bwd::Params p;
   p.lse = lse;
-  p.delta = reinterpret_cast<const float *>(workspace);
+  p.delta = reinterpret_cast<float *>(workspace);
+  p.o = reinterpret_cast<const uint16_t *>(o);
   p.dq = reinterpret_cast<uint16_t *>(dq);
   p.dk = reinterpret_cast<uint16_t *>(dk);
   p.dv = reinterpret_cast<uint16_t *>(dv);
@@ -897,7 +971,8 @@ int mk_attn_bwd(const void *q, const void *k, const void *v, const void *o, cons
                 int D, int causal, float scale, const int32_t *cu_seqlens, void *workspace,
                 int64_t workspace_bytes, void *stream) {
   return mk_attn_bwd_stages(q, k, v, o, lse, dO, dq, dk, dv, B, Hq, Hkv, S, D, causal, scale,
-                            cu_seqlens, workspace, workspace_bytes, MK_BWD_ALL, stream);
+                            cu_seqlens, workspace, workspace_bytes, MK_BWD_DQ | MK_BWD_DKDV,
+                            stream);
 }
 
 }  // extern "C"
