@@ -314,6 +314,13 @@ MK_API int mk_attn_mla_decode_paged(const void *q, const void *cache, const int3
 #define MK_SCHED_SNAKE 0       /* round k: CTA c takes unit kG + c, or kG + G-1-c in odd rounds */
 #define MK_SCHED_ROUND_ROBIN 1 /* round k: CTA c takes unit kG + c */
 #define MK_SCHED_BLOCKED 2     /* CTA c takes units c*ceil(n/G) .. (c+1)*ceil(n/G) - 1 */
+#define MK_SCHED_DYNAMIC 3     /* forward: CTA c takes unit c, then claims the next
+                                  unclaimed unit from a device counter shortly before
+                                  each of its units ends (greedy, heaviest first).  The
+                                  counters are a ring of 1024 per device, one per launch,
+                                  reset by each launch's last CTA: at most 1024 forward
+                                  launches may execute at once on a device.  The
+                                  backward kernels take it as MK_SCHED_SNAKE. */
 
 /*
  * Launch parameters that change speed but never results beyond rounding:

@@ -29,7 +29,7 @@ FLUSH_BYTES = 256 << 20
 SPACES = {
     "prefill": dict(ctas=[0, 148, 144, 136, 128, 114, 76],
                     schedule=[binding.SCHED_SNAKE, binding.SCHED_ROUND_ROBIN,
-                              binding.SCHED_BLOCKED],
+                              binding.SCHED_BLOCKED, binding.SCHED_DYNAMIC],
                     rescale_log2=[0.0, 4.0, 8.0, 12.0]),
     "backward": dict(ctas=[0, 148, 136, 114],
                      schedule=[binding.SCHED_SNAKE, binding.SCHED_ROUND_ROBIN,

@@ -28,7 +28,7 @@ BWD_DELTA, BWD_DKDV, BWD_DQ, BWD_ALL = 1, 2, 4, 7
 MLA_DQK, MLA_DV = 576, 512
 
 # Unit schedules (MK_SCHED_*).
-SCHED_SNAKE, SCHED_ROUND_ROBIN, SCHED_BLOCKED = 0, 1, 2
+SCHED_SNAKE, SCHED_ROUND_ROBIN, SCHED_BLOCKED, SCHED_DYNAMIC = 0, 1, 2, 3
 
 
 class MkAttnTuning(ctypes.Structure):

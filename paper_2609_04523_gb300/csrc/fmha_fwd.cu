@@ -75,6 +75,12 @@ constexpr int kCuCache = 2048;        // cu_seqlens entries cached in shared mem
 constexpr int kMaxLevels = 1024;      // causal varlen: longest-first order up to 1024 tile pairs
                                       // (262144 tokens) per sequence
 
+// MK_SCHED_DYNAMIC: per-launch claim counter and finished-CTA counter, a ring
+// of slots so that launches running at once on other streams do not share
+// one.  Zero at load; each launch's last CTA puts its slot back to zero.
+constexpr int kSchedSlots = 1024;
+__device__ unsigned g_sched_next[kSchedSlots];
+__device__ unsigned g_sched_done[kSchedSlots];
 __device__ int g_status = 0;               // MK_ERR_TIMEOUT once a wait ran out
 
 template <int D>
@@ -135,6 +141,7 @@ struct Params {
   int stall_first_slot;     // failure-path test: the producer loads nothing
   int schedule;             // MK_SCHED_*: units over the persistent CTAs
   float rescale_log2;       // lazy O rescale threshold (log2 units)
+  int sched_slot;           // MK_SCHED_DYNAMIC: this launch's counter slot
 };
 
 __device__ __forceinline__ int clamp_tok(int x, int T) { return x < 0 ? 0 : (x > T ? T : x); }
@@ -304,6 +311,17 @@ __device__ __forceinline__ int unit_of_round(int k, int schedule, int n_units) {
   return (k & 1) ? (k + 1) * G - 1 - c : k * G + c;
 }
 
+// MK_SCHED_DYNAMIC, at CTA exit (one thread, after the CTA's last claim): the
+// launch's last CTA puts its counter slot back to zero.  Out of line, so that
+// nothing of it is held in registers across the kernel.
+__device__ __noinline__ void sched_release(int slot) {
+  __threadfence();
+  if (atomicAdd(&g_sched_done[slot], 1u) == gridDim.x - 1) {
+    atomicExch(&g_sched_next[slot], 0u);
+    atomicExch(&g_sched_done[slot], 0u);
+  }
+}
+
 // Bounded wait that ignores the abort flag: used only at teardown to let
 // operations already in flight land before the CTA releases its resources.
 __device__ __forceinline__ void drain_wait(uint64_t *bar, uint32_t parity) {
@@ -422,10 +440,29 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         ++n_pub;
       };
+      // MK_SCHED_DYNAMIC: the first unit is blockIdx.x; each later one is
+      // claimed (lane 0) two key blocks before the current unit's loads end,
+      // and the claim's result is read at the next unit, so its latency is
+      // hidden.  A unit without a claim point claims at the top of the loop.
+      unsigned claim = 0;
+      bool claimed = false;
       bool ok = true;
-      for (int k = 0; ok && k * (int)gridDim.x < p.n_units; ++k) {
-        const int u = unit_of_round(k, p.schedule, p.n_units);
-        if (u >= p.n_units) continue;
+      for (int k = 0; ok; ++k) {
+        int u;
+        if (p.schedule == MK_SCHED_DYNAMIC) {
+          if (k == 0) {
+            u = blockIdx.x;
+          } else {
+            if (!claimed && lane_id() == 0) claim = atomicAdd(&g_sched_next[p.sched_slot], 1u);
+            u = (int)gridDim.x + (int)__shfl_sync(0xffffffffu, claim, 0);
+            claimed = false;
+          }
+          if (u >= p.n_units) break;
+        } else {
+          if (k * (int)gridDim.x >= p.n_units) break;
+          u = unit_of_round(k, p.schedule, p.n_units);
+          if (u >= p.n_units) continue;
+        }
         const Unit w = map_unit<VL>(p, cu_smem, sched, u);
         if (!w.valid) continue;
         publish(w);
@@ -452,7 +489,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         };
         load_q(0);
         if (!ok) break;
+        const int claim_j = n_blk > 2 ? n_blk - 2 : 0;
         for (int j = 0; j <= n_blk; ++j) {
+          if (p.schedule == MK_SCHED_DYNAMIC && j == claim_j) {
+            if (lane_id() == 0) claim = atomicAdd(&g_sched_next[p.sched_slot], 1u);
+            claimed = true;
+          }
           const int s = it % NS;
           ok = mbar_wait_all(&ctl->bar_kv_empty[s], ((it / NS) & 1) ^ 1, abort);
           if (!ok) break;
@@ -833,6 +875,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0 && ctl->abort) {
     atomicExch(&g_status, (int)MK_ERR_TIMEOUT);
   }
+  // MK_SCHED_DYNAMIC: every claim of this CTA was made before the barrier
+  // above; the launch's last CTA to finish puts the slot back to zero.
+  if (p.schedule == MK_SCHED_DYNAMIC && threadIdx.x == 0) sched_release(p.sched_slot);
 }
 
 // =================================================================== host
@@ -947,6 +992,8 @@ static int attn_fwd_impl(const void *q, const void *k, const void *v, void *o, f
   const mk_attn_tuning tune = current_tuning();
   p.schedule = tune.schedule;
   p.rescale_log2 = tune.rescale_log2;
+  static std::atomic<uint32_t> sched_epoch{0};
+  p.sched_slot = (int)(sched_epoch.fetch_add(1, std::memory_order_relaxed) % kSchedSlots);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (D == 128)
     return varlen ? launch<128, true>(q, k, v, p, tokens, st) : launch<128, false>(q, k, v, p, tokens, st);

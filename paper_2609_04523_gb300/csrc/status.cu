@@ -52,7 +52,7 @@ int mk_attn_set_tuning(const mk_attn_tuning *t) {
   mk_attn_tuning v = mk::kDefaultTuning;
   if (t) {
     if (t->ctas < 0 || t->ctas > 65535) return MK_ERR_INVALID_ARG;
-    if (t->schedule < MK_SCHED_SNAKE || t->schedule > MK_SCHED_BLOCKED) return MK_ERR_INVALID_ARG;
+    if (t->schedule < MK_SCHED_SNAKE || t->schedule > MK_SCHED_DYNAMIC) return MK_ERR_INVALID_ARG;
     if (!(t->rescale_log2 >= 0.0f && t->rescale_log2 <= 16.0f)) return MK_ERR_INVALID_ARG;
     if (t->split_ctas_per_sm < 1 || t->split_ctas_per_sm > 64) return MK_ERR_INVALID_ARG;
     if (t->split_min_pages < 1 || t->split_min_pages > 4096) return MK_ERR_INVALID_ARG;

@@ -19,7 +19,7 @@ def test_defaults():
 
 
 @pytest.mark.parametrize("field, bad", [
-    ("ctas", -1), ("ctas", 65536), ("schedule", -1), ("schedule", 3),
+    ("ctas", -1), ("ctas", 65536), ("schedule", -1), ("schedule", 4),
     ("rescale_log2", -0.5), ("rescale_log2", 16.5), ("rescale_log2", float("nan")),
     ("split_ctas_per_sm", 0), ("split_ctas_per_sm", 65), ("split_min_pages", 0),
     ("split_min_pages", 4097), ("mla_split_ctas_per_sm", 0), ("mla_split_ctas_per_sm", 65)])

@@ -37,7 +37,9 @@ def check_fwd(o, lse, o_ref, lse_ref):
 
 
 KNOBS = [dict(ctas=1), dict(ctas=37), dict(ctas=300), dict(schedule=binding.SCHED_ROUND_ROBIN),
-         dict(schedule=binding.SCHED_BLOCKED), dict(ctas=64, schedule=binding.SCHED_BLOCKED)]
+         dict(schedule=binding.SCHED_BLOCKED), dict(ctas=64, schedule=binding.SCHED_BLOCKED),
+         dict(schedule=binding.SCHED_DYNAMIC), dict(ctas=1, schedule=binding.SCHED_DYNAMIC),
+         dict(ctas=37, schedule=binding.SCHED_DYNAMIC)]
 
 
 @pytest.mark.parametrize("knob", KNOBS, ids=lambda d: "-".join(f"{k}{v}" for k, v in d.items()))
@@ -145,3 +147,32 @@ def test_sweep_returns_sorted_rows_and_restores_tuning():
     assert len(rows) == 4 and all(r["ms"] > 0 for r in rows)
     assert rows == sorted(rows, key=lambda r: r["ms"])
     assert binding.mk_attn_get_tuning().ctas == 99
+
+
+def test_dynamic_schedule_counters_reset_over_many_launches_and_two_streams():
+    """MK_SCHED_DYNAMIC claims units from per-launch device counters that each
+    launch's last CTA zeroes.  1100 launches wrap the 1024-slot ring, so every
+    slot is reused; launches alternate between two streams so that some run at
+    once.  Every output must equal the snake schedule's bit for bit (a counter
+    left non-zero would skip units)."""
+    dev = torch.device("cuda")
+    q, k, v, _ = W.make_qkv(1, 4, 2, 2048, 64, seed=932)
+    q, k, v = q.to(dev), k.to(dev), v.to(dev)
+    o_ref, lse_ref = binding.attn_fwd(q, k, v, causal=True, scale=0.125)
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    for st in streams:
+        st.wait_stream(torch.cuda.current_stream())
+    outs = []
+    with binding.tuning(ctas=5, schedule=binding.SCHED_DYNAMIC):
+        for i in range(1100):
+            st = streams[i % 2]
+            with torch.cuda.stream(st):
+                o = torch.empty_like(q)
+                lse = torch.empty((1, 4, 2048), dtype=torch.float32, device=dev)
+                binding.attn_fwd(q, k, v, causal=True, scale=0.125, out=o, lse=lse, stream=st)
+            if i % 50 == 0 or i >= 1090:
+                outs.append((st, o, lse))
+        torch.cuda.synchronize()
+    assert binding.mk_attn_check_status(torch.cuda.current_stream().cuda_stream) == 0
+    for _, o, lse in outs:
+        assert torch.equal(o, o_ref) and torch.equal(lse, lse_ref)
