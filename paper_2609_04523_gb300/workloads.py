@@ -93,6 +93,17 @@ def varlen_lengths(seed: int, total: int, lo: int = 512, hi: int = 4096) -> list
     return lens
 
 
+def many_short_lengths(n: int, seed: int) -> list[int]:
+    """n lengths drawn uniformly from 0..39 (empty sequences included), with a
+    300-token sequence at index n - 50 and a 129-token one last, when n > 50."""
+    rng = np.random.default_rng(seed)
+    lens = [int(x) for x in rng.integers(0, 40, size=n)]
+    if n > 50:
+        lens[n - 50] = 300
+        lens[n - 1] = 129
+    return lens
+
+
 def cu_from_lengths(lens) -> torch.Tensor:
     cu = [0]
     for L in lens:

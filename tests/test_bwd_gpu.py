@@ -91,6 +91,15 @@ def test_bwd_varlen(causal, D):
     check(q, k, v, do, causal, 1.0 / math.sqrt(D), cu=cu, what=f"varlen D{D} causal={causal}")
 
 
+def test_bwd_varlen_more_sequences_than_one_warp_scan():
+    """2100 packed sequences, empty ones among them: the backward kernels find a
+    unit's sequence by warp scans over cu_seqlens in chunks of 32 sequences."""
+    lens = W.many_short_lengths(2100, seed=92)
+    q, k, v, cu = W.make_qkv(0, 4, 2, 0, 64, seed=92, lengths=lens)
+    do = W.make_grad_out(q.shape, seed=92)
+    check(q, k, v, do, True, 0.125, cu=cu, what="varlen 2100 sequences")
+
+
 @pytest.mark.parametrize("scale", [-0.09, 0.0, 0.3])
 def test_bwd_scales(scale):
     """Negative, zero and large scales (zero scale: dq = dk = 0)."""

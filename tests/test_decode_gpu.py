@@ -74,6 +74,15 @@ def test_decode_splits(B):
     check(inp, f"B{B}")
 
 
+def test_decode_many_sequences():
+    """3000 sequences of 0..199 cached keys (page 16): one split each for most,
+    a grid of 3000 sequences in z, empty sequences among them."""
+    rng = np.random.default_rng(715)
+    lens = [int(x) for x in rng.integers(0, 200, size=3000)]
+    inp = W.make_paged(lens, 8, 2, 128, 16, seed=715)
+    check(inp, "B3000")
+
+
 def test_decode_uneven_lengths_with_empty_splits():
     """One long sequence sets max_pages; the short ones leave most of their
     splits empty (lse -inf partials), which the merge must ignore."""

@@ -65,6 +65,15 @@ def test_mla_splits(B):
     check(inp, f"B{B}")
 
 
+def test_mla_many_sequences():
+    """600 sequences of 0..299 latent rows (page 16, 16 heads): a grid of 1200
+    value-half CTAs per split, empty sequences among them."""
+    rng = np.random.default_rng(985)
+    lens = [int(x) for x in rng.integers(0, 300, size=600)]
+    inp = W.make_mla_paged(lens, 16, 16, seed=985)
+    check(inp, "B600")
+
+
 def test_mla_large_logits():
     """Row maxima that rise by far more than the lazy-rescale threshold
     between blocks (q and cache ~ N(0, 4))."""

@@ -143,6 +143,19 @@ def test_varlen_with_empty_sequences():
     assert_close(o, lse, o_ref, lse_ref, "varlen empty sequences")
 
 
+@pytest.mark.parametrize("causal", [True, False])
+def test_varlen_more_sequences_than_cu_cache(causal):
+    """2100 packed sequences: the kernel caches cu_seqlens[0..2047] in shared
+    memory and reads the entries past it from global memory.  Lengths 0..39,
+    with a 300- and a 129-token sequence past the cache, so ragged tiles and
+    empty sequences occur on both sides of it."""
+    lens = W.many_short_lengths(2100, seed=91)
+    q, k, v, cu = W.make_qkv(0, 4, 2, 0, 64, seed=91, lengths=lens)
+    o, lse = gpu_attn(q, k, v, causal, 0.125, cu)
+    o_ref, lse_ref = oracle.attn_fwd(q, k, v, causal, 0.125, cu_seqlens=cu.numpy())
+    assert_close(o, lse, o_ref, lse_ref, "varlen 2100 sequences")
+
+
 # ----------------------------------------------------------- special cases
 
 def test_zero_scale_gives_prefix_means():
