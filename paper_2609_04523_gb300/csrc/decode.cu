@@ -448,18 +448,42 @@ __global__ void __launch_bounds__(128) merge_kernel(const Params p) {
   L = L < 0 ? 0 : (L > p.max_pages * p.page_size ? p.max_pages * p.page_size : L);
   const int n_pages = (L + p.page_size - 1) / p.page_size;
   const int n_valid = max(1, min(p.n_splits, (n_pages + p.pages_per_split - 1) / p.pages_per_split));
+  // The split lse values, one per lane, then a warp max: the loads are issued
+  // together rather than one after another.
   float mx = -INFINITY;
-  for (int s = 0; s < n_valid; ++s) mx = fmaxf(mx, pr[s * (D + 1) + D]);
+  for (int s0 = 0; s0 < n_valid; s0 += 32) {
+    const int s = s0 + lane;
+    mx = fmaxf(mx, s < n_valid ? pr[s * (D + 1) + D] : -INFINITY);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
   float acc[NDL];
 #pragma unroll
   for (int e = 0; e < NDL; ++e) acc[e] = 0.f;
   float wsum = 0.f;
   if (mx > -INFINITY) {
-    for (int s = 0; s < n_valid; ++s) {
-      const float w = exp2f((pr[s * (D + 1) + D] - mx) * 1.4426950408889634f);
-      wsum += w;
+    // Groups of kGroup splits: every load of a group is issued before the
+    // first use; the sums run in split order.
+    constexpr int kGroup = 8;
+    for (int s0 = 0; s0 < n_valid; s0 += kGroup) {
+      float lv[kGroup], v[kGroup][NDL];
 #pragma unroll
-      for (int e = 0; e < NDL; ++e) acc[e] = fmaf(w, pr[s * (D + 1) + lane * NDL + e], acc[e]);
+      for (int t = 0; t < kGroup; ++t) {
+        const bool in = s0 + t < n_valid;
+        const float *ps = pr + (int64_t)(s0 + t) * (D + 1);
+        lv[t] = in ? ps[D] : -INFINITY;
+#pragma unroll
+        for (int e = 0; e < NDL; ++e) v[t][e] = in ? ps[lane * NDL + e] : 0.f;
+      }
+#pragma unroll
+      for (int t = 0; t < kGroup; ++t) {
+        if (s0 + t < n_valid) {
+          const float w = exp2f((lv[t] - mx) * 1.4426950408889634f);
+          wsum += w;
+#pragma unroll
+          for (int e = 0; e < NDL; ++e) acc[e] = fmaf(w, v[t][e], acc[e]);
+        }
+      }
     }
   }
   const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
