@@ -78,7 +78,8 @@ typedef enum {
  * descriptors and enqueues one kernel on `stream`; it returns without
  * synchronising.  On any error it returns a negative mk_status and enqueues
  * nothing, so o and lse are left untouched.  The library allocates no device
- * memory.  Results are deterministic: no atomics, so repeated calls on the same
+ * memory.  Results are deterministic: each output element is computed by one
+ * CTA in a fixed order, under every schedule, so repeated calls on the same
  * inputs are bitwise identical.  Sequences of length 0 (varlen) produce no
  * rows.  Every internal wait of the kernel is bounded; if one runs out the
  * kernel records MK_ERR_TIMEOUT for mk_attn_check_status and exits.
