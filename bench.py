@@ -281,6 +281,63 @@ def job_tflops(flops_per_rank: float, steps: int, job_ms: float, world: int) -> 
     return world * flops_per_rank * steps / (job_ms * 1e-3) / 1e12
 
 
+E2E_PIPELINED = ("pipelined: every step copies its inputs from pinned host memory and its "
+                 "outputs back; two device buffer sets, the inputs of step i+1 copied on one "
+                 "stream while step i computes, the outputs of step i copied back on another "
+                 "while step i+1 computes")
+
+
+def e2e_pipelined(steps: int, stream, dev, hosts_in, devs_in, hosts_out, devs_out, call) -> float:
+    """Milliseconds for `steps` end-to-end steps with the copies overlapped.
+
+    Step i uses device buffer set b = i % 2 (devs_in[b], devs_out[b]): its
+    inputs are copied from `hosts_in` on an input stream, `call(b)` runs on
+    `stream`, and its outputs are copied to `hosts_out` on an output stream.
+    Events order the reuse of a set: step i's input copy waits for the call of
+    step i - 2 (which read that set), and step i's call waits for the output
+    copy of step i - 2.  The region runs from an event on `stream` before the
+    first copy to one after the last output copy."""
+    import torch
+    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    ev_in = [torch.cuda.Event() for _ in range(2)]
+    ev_call = [torch.cuda.Event() for _ in range(2)]
+    ev_out = [torch.cuda.Event() for _ in range(2)]
+
+    def run(n):
+        for i in range(n):
+            b = i % 2
+            if i >= 2:
+                s_in.wait_event(ev_call[b])
+            with torch.cuda.stream(s_in):
+                for d_, h_ in zip(devs_in[b], hosts_in):
+                    d_.copy_(h_, non_blocking=True)
+            ev_in[b].record(s_in)
+            stream.wait_event(ev_in[b])
+            if i >= 2:
+                stream.wait_event(ev_out[b])
+            call(b)
+            ev_call[b].record(stream)
+            s_out.wait_event(ev_call[b])
+            with torch.cuda.stream(s_out):
+                for h_, d_ in zip(hosts_out, devs_out[b]):
+                    h_.copy_(d_, non_blocking=True)
+            ev_out[b].record(s_out)
+        stream.wait_stream(s_in)
+        stream.wait_stream(s_out)
+
+    torch.cuda.synchronize(dev)
+    run(2)  # warm-up
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    s_in.wait_event(e0)
+    s_out.wait_event(e0)
+    run(steps)
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    return e0.elapsed_time(e1)
+
+
 def run_ours(args, rank: int, world: int, local_rank: int):
     import numpy as np
     import torch
@@ -381,7 +438,24 @@ def run_ours(args, rank: int, world: int, local_rank: int):
         e2e_step()
     e1.record(stream)
     torch.cuda.synchronize(dev)
-    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    serial_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    serial_tflops = job_tflops(flops, args.steps, serial_ms, world)
+    # The same steps with the copies overlapped (second buffer set).
+    sets_in = [[qd, kd, vd] + ([] if cud is None else [cud])]
+    sets_in.append([torch.empty_like(t) for t in sets_in[0]])
+    sets_out = [[o, lse], [torch.empty_like(o), torch.empty_like(lse)]]
+    hosts = [qh, kh, vh] + ([] if cuh is None else [cuh])
+
+    def call(b):
+        qb, kb, vb = sets_in[b][:3]
+        cub = sets_in[b][3] if cud is not None else None
+        attn_fwd(qb, kb, vb, c.causal, c.scale, cub, out=sets_out[b][0], lse=sets_out[b][1],
+                 stream=stream)
+
+    if world > 1:
+        torch.distributed.barrier()
+    e2e_ms = max_over_ranks(e2e_pipelined(args.steps, stream, dev, hosts, sets_in, [oh, lh],
+                                          sets_out, call), world, dev)
     e2e_tflops = job_tflops(flops, args.steps, e2e_ms, world)
 
     if rank != 0:
@@ -424,7 +498,9 @@ def run_ours(args, rank: int, world: int, local_rank: int):
             "kernel": f"mk::fmha_fwd_kernel<{c.D}>",
         },
         "e2e": {"value": round(e2e_tflops, 2), "unit": "TFLOP/s",
-                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "mode": E2E_PIPELINED,
+                "serial_value": round(serial_tflops, 2),
+                "serial_mode": "copy in, call, copy out, all on the call's stream"},
         "gpu_launches": args.steps,
         "clocks": clocks,
     }
@@ -578,7 +654,20 @@ def run_decode(args, rank: int, world: int, local_rank: int):
         e2e_step()
     e1.record(stream)
     torch.cuda.synchronize(dev)
-    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    serial_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    serial_gbs = world * nbytes * args.steps / (serial_ms * 1e-3) / 1e9
+    # The same steps with the copies overlapped (second buffer set).
+    sets_in = [[qd, ptd, sld], [torch.empty_like(qd), torch.empty_like(ptd), torch.empty_like(sld)]]
+    sets_out = [[o, lse], [torch.empty_like(o), torch.empty_like(lse)]]
+
+    def call(b):
+        decode_paged(sets_in[b][0], kc, vc, sets_in[b][1], sets_in[b][2], inp.scale,
+                     out=sets_out[b][0], lse=sets_out[b][1], workspace=ws, stream=stream)
+
+    if world > 1:
+        torch.distributed.barrier()
+    e2e_ms = max_over_ranks(e2e_pipelined(args.steps, stream, dev, [qh, pth, slh], sets_in,
+                                          [oh, lh], sets_out, call), world, dev)
     e2e_gbs = world * nbytes * args.steps / (e2e_ms * 1e-3) / 1e9
 
     if rank != 0:
@@ -620,7 +709,9 @@ def run_decode(args, rank: int, world: int, local_rank: int):
             "kernel": "mk::dec::decode_kernel<128, 4>" + (" + merge_kernel<128>" if need > 0 else ""),
         },
         "e2e": {"value": round(e2e_gbs, 1), "unit": "GB/s",
-                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "mode": E2E_PIPELINED,
+                "serial_value": round(serial_gbs, 1),
+                "serial_mode": "copy in, call, copy out, all on the call's stream"},
         "gpu_launches": args.steps * launches,
         "clocks": clocks,
     }
@@ -822,7 +913,23 @@ def run_backward(args, rank: int, world: int, local_rank: int):
         e2e_step()
     e1.record(stream)
     torch.cuda.synchronize(dev)
-    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    serial_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    serial_tflops = job_tflops(flops, args.steps, serial_ms, world)
+    # The same steps with the copies overlapped (second buffer set).
+    sets_in = [devs_in, [torch.empty_like(t) for t in devs_in]]
+    sets_out = [[dq, dk, dv], [torch.empty_like(dq), torch.empty_like(dk), torch.empty_like(dv)]]
+
+    def call(b):
+        di = sets_in[b]
+        cub = di[6] if inp.cu_seqlens is not None else None
+        attn_bwd(di[0], di[1], di[2], di[3], di[4], di[5], c.causal, c.scale, cub,
+                 dq=sets_out[b][0], dk=sets_out[b][1], dv=sets_out[b][2], workspace=ws,
+                 stream=stream)
+
+    if world > 1:
+        torch.distributed.barrier()
+    e2e_ms = max_over_ranks(e2e_pipelined(args.steps, stream, dev, hosts_in, sets_in, hosts_out,
+                                          sets_out, call), world, dev)
     e2e_tflops = job_tflops(flops, args.steps, e2e_ms, world)
 
     if rank != 0:
@@ -868,7 +975,9 @@ def run_backward(args, rank: int, world: int, local_rank: int):
             "dq_kernel_tflops_executed": round(dq_tflops, 2),
         },
         "e2e": {"value": round(e2e_tflops, 2), "unit": "TFLOP/s",
-                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "mode": E2E_PIPELINED,
+                "serial_value": round(serial_tflops, 2),
+                "serial_mode": "copy in, call, copy out, all on the call's stream"},
         "gpu_launches": 2 * args.steps,
         "clocks": clocks,
     }
@@ -1058,7 +1167,21 @@ def run_mla(args, rank: int, world: int, local_rank: int):
         e2e_step()
     e1.record(stream)
     torch.cuda.synchronize(dev)
-    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    serial_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    serial_gbs = world * nbytes * args.steps / (serial_ms * 1e-3) / 1e9
+    # The same steps with the copies overlapped (second buffer set).
+    sets_in = [[qd, ptd, sld], [torch.empty_like(qd), torch.empty_like(ptd), torch.empty_like(sld)]]
+    sets_out = [[o, lse], [torch.empty_like(o), torch.empty_like(lse)]]
+
+    def call(b):
+        binding.mla_decode_paged(sets_in[b][0], c, sets_in[b][1], sets_in[b][2], inp.scale,
+                                 out=sets_out[b][0], lse=sets_out[b][1], workspace=ws,
+                                 stream=stream)
+
+    if world > 1:
+        torch.distributed.barrier()
+    e2e_ms = max_over_ranks(e2e_pipelined(args.steps, stream, dev, [qh, pth, slh], sets_in,
+                                          [oh, lh], sets_out, call), world, dev)
     e2e_gbs = world * nbytes * args.steps / (e2e_ms * 1e-3) / 1e9
 
     if rank != 0:
@@ -1103,7 +1226,9 @@ def run_mla(args, rank: int, world: int, local_rank: int):
             "kernel": "mk::mla::mla_decode_kernel" + (" + mla_merge_kernel" if need > 0 else ""),
         },
         "e2e": {"value": round(e2e_gbs, 1), "unit": "GB/s",
-                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "mode": E2E_PIPELINED,
+                "serial_value": round(serial_gbs, 1),
+                "serial_mode": "copy in, call, copy out, all on the call's stream"},
         "gpu_launches": args.steps * launches,
         "clocks": clocks,
     }
