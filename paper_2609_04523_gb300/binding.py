@@ -271,10 +271,10 @@ def attn_bwd(q, k, v, o, lse, do, causal: bool = True, scale: float | None = Non
 
     q, k, v, causal, scale, cu_seqlens as for attn_fwd; o, lse its outputs;
     do: bf16 gradient of o (layout of q).  Returns (dq, dk, dv), bf16, the
-    layouts of q, k, v.  `stages` (BWD_* flags) enqueues only some of the three
-    kernels; dK/dV and dQ need the Delta an earlier call wrote into the same
-    `workspace`.  PyTorch only allocates the outputs and the fp32 workspace and
-    provides the stream."""
+    layouts of q, k, v.  `stages` (BWD_* flags) enqueues only some stages:
+    BWD_DQ computes Delta itself and writes it to `workspace`; BWD_DKDV reads
+    the Delta an earlier BWD_DQ or BWD_DELTA stage wrote there.  PyTorch only
+    allocates the outputs and the fp32 workspace and provides the stream."""
     import torch
     for name, t in (("q", q), ("k", k), ("v", v), ("o", o), ("do", do)):
         if not t.is_cuda or t.dtype != torch.bfloat16 or not t.is_contiguous():

@@ -100,6 +100,50 @@ def test_bwd_varlen_more_sequences_than_one_warp_scan():
     check(q, k, v, do, True, 0.125, cu=cu, what="varlen 2100 sequences")
 
 
+@pytest.mark.parametrize("causal", [True, False])
+def test_bwd_stages_separately(causal):
+    """mk_attn_bwd_stages: dQ alone (which writes Delta into the workspace),
+    then dK/dV alone, equal the full call bit for bit; the stand-alone Delta
+    kernel followed by dK/dV meets the oracle (its Delta sums in another order,
+    so not bitwise).  Outputs of stages not enqueued stay untouched."""
+    dev = torch.device("cuda")
+    lens = [300, 1, 129, 700]
+    q, k, v, cu = W.make_qkv(0, 8, 2, 0, 128, seed=893 + int(causal), lengths=lens)
+    do = W.make_grad_out(q.shape, seed=893)
+    qd, kd, vd, dod, cud = q.to(dev), k.to(dev), v.to(dev), do.to(dev), cu.to(dev)
+    o, lse = binding.attn_fwd(qd, kd, vd, causal=causal, scale=0.09, cu_seqlens=cud)
+    need = binding.mk_attn_bwd_workspace_bytes(len(lens), 8, q.shape[0], True)
+    ws = torch.empty((need + 15) // 16 * 4, dtype=torch.float32, device=dev)
+
+    def nan_outputs():
+        return (torch.full_like(qd, float("nan")), torch.full_like(kd, float("nan")),
+                torch.full_like(vd, float("nan")))
+
+    def run(stages, outs):
+        binding.attn_bwd(qd, kd, vd, o, lse, dod, causal=causal, scale=0.09, cu_seqlens=cud,
+                         dq=outs[0], dk=outs[1], dv=outs[2], workspace=ws, stages=stages)
+        assert binding.mk_attn_check_status(torch.cuda.current_stream().cuda_stream) == 0
+
+    full = nan_outputs()
+    run(binding.BWD_ALL, full)
+    sep = nan_outputs()
+    run(binding.BWD_DQ, sep)
+    assert torch.isnan(sep[1].float()).all() and torch.isnan(sep[2].float()).all()
+    assert torch.equal(sep[0], full[0])
+    run(binding.BWD_DKDV, sep)
+    assert torch.equal(sep[1], full[1]) and torch.equal(sep[2], full[2])
+
+    ws.fill_(float("nan"))
+    via_delta = nan_outputs()
+    run(binding.BWD_DELTA, via_delta)
+    assert all(torch.isnan(t.float()).all() for t in via_delta)
+    run(binding.BWD_DKDV, via_delta)
+    assert torch.isnan(via_delta[0].float()).all()
+    _, rk, rv = oracle.attn_bwd(q, k, v, do, causal, 0.09, cu_seqlens=cu.numpy())
+    compare(via_delta[1].float().cpu().numpy(), rk, "Delta kernel + dK/dV: dk")
+    compare(via_delta[2].float().cpu().numpy(), rv, "Delta kernel + dK/dV: dv")
+
+
 @pytest.mark.parametrize("scale", [-0.09, 0.0, 0.3])
 def test_bwd_scales(scale):
     """Negative, zero and large scales (zero scale: dq = dk = 0)."""
