@@ -320,7 +320,9 @@ MK_API int mk_attn_mla_decode_paged(const void *q, const void *cache, const int3
                                   each of its units ends (greedy, heaviest first).  The
                                   counters are a ring of 1024 per device, one per launch,
                                   reset by each launch's last CTA: at most 1024 forward
-                                  launches may execute at once on a device.  The
+                                  launches may execute at once on a device.  A launch
+                                  captured in a CUDA graph keeps its slot, so two
+                                  instances of that graph must not run at once.  The
                                   backward kernels take it as MK_SCHED_SNAKE. */
 
 /*
