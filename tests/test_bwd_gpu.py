@@ -74,7 +74,7 @@ def test_bwd_fixed_length(D, causal, S):
     check(q, k, v, do, causal, 1.0 / math.sqrt(D), what=f"S{S} D{D} causal={causal}")
 
 
-@pytest.mark.parametrize("G", [1, 4, 8])
+@pytest.mark.parametrize("G", [1, 4, 8, 16])
 def test_bwd_group_sizes(G):
     q, k, v, _ = W.make_qkv(1, 2 * G, 2, 640, 128, seed=850 + G)
     do = W.make_grad_out(q.shape, seed=850 + G)

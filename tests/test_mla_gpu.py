@@ -50,6 +50,14 @@ def test_mla_lengths(page_size, Hq):
     check(inp, f"ps{page_size} Hq{Hq}")
 
 
+@pytest.mark.parametrize("Hq", [1, 129])
+def test_mla_one_head_and_one_past_a_group(Hq):
+    """One head (127 zero-filled rows of the M = 128 tile), and 129 heads (a
+    second group holding a single head)."""
+    inp = W.make_mla_paged([0, 1, 300, 1500], Hq, 64, seed=975 + Hq)
+    check(inp, f"Hq{Hq}")
+
+
 def test_mla_two_head_groups():
     """200 heads: a full group of 128 and a partial one of 72."""
     inp = W.make_mla_paged([300, 1500], 200, 64, seed=971)

@@ -95,6 +95,12 @@ def test_gqa_groups(D, G, B):
 
 
 @pytest.mark.parametrize("causal", [True, False])
+def test_mqa_one_kv_head_for_64_query_heads(causal):
+    """Multi-query attention: G = 64, every query head reads key/value head 0."""
+    check_fixed(B=1, Hq=64, Hkv=1, S=300, D=128, causal=causal, seed=170 + int(causal))
+
+
+@pytest.mark.parametrize("causal", [True, False])
 def test_gqa_odd_group(causal):
     """G = 3: units pair consecutive row tiles of one head (no head pairs)."""
     check_fixed(B=2, Hq=6, Hkv=2, S=700, D=128, causal=causal, seed=150 + int(causal))
