@@ -74,6 +74,13 @@ def test_decode_splits(B):
     check(inp, f"B{B}")
 
 
+def test_decode_one_long_sequence():
+    """One sequence of 131072 cached keys (2048 pages of 64): every split of the
+    plan belongs to it, and the merge combines them all."""
+    inp = W.make_paged([131072], 8, 2, 128, 64, seed=716)
+    check(inp, "L131072")
+
+
 def test_decode_many_sequences():
     """3000 sequences of 0..199 cached keys (page 16): one split each for most,
     a grid of 3000 sequences in z, empty sequences among them."""

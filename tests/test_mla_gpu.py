@@ -58,6 +58,13 @@ def test_mla_one_head_and_one_past_a_group(Hq):
     check(inp, f"Hq{Hq}")
 
 
+def test_mla_one_long_sequence():
+    """One sequence of 65536 latent rows (1024 pages of 64), 128 heads: all the
+    KV splits belong to it."""
+    inp = W.make_mla_paged([65536], 128, 64, seed=977)
+    check(inp, "L65536")
+
+
 def test_mla_two_head_groups():
     """200 heads: a full group of 128 and a partial one of 72."""
     inp = W.make_mla_paged([300, 1500], 200, 64, seed=971)
