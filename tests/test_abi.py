@@ -86,3 +86,79 @@ def test_missing_library_fails_loudly(monkeypatch, tmp_path):
     monkeypatch.setattr(binding, "LIB_PATH", str(tmp_path / "absent.so"))
     with pytest.raises(binding.MkAttnError):
         binding.load_library()
+
+
+# The other entry points check their arguments on the host before their first
+# CUDA call too, so these rejections need no GPU.  (Checks that depend on the
+# device -- the decode split plan's workspace size -- are covered by the GPU
+# tests.)
+BWD_GOOD = dict(q=A, k=2 * A, v=3 * A, o=4 * A, lse=5 * A, do=6 * A, dq=7 * A, dk=8 * A,
+                dv=9 * A, B=2, Hq=8, Hkv=2, S=256, D=128, causal=1, scale=0.088,
+                cu_seqlens=None, workspace=10 * A, workspace_bytes=2 * 8 * 256 * 4,
+                stages=binding.BWD_ALL, stream=None)
+
+
+@pytest.mark.parametrize("kw, want", [
+    (dict(stages=0), binding.MK_ERR_INVALID_ARG),
+    (dict(stages=8), binding.MK_ERR_INVALID_ARG),
+    (dict(do=None), binding.MK_ERR_INVALID_ARG),
+    (dict(dv=None), binding.MK_ERR_INVALID_ARG),
+    (dict(workspace=None), binding.MK_ERR_INVALID_ARG),
+    (dict(Hkv=3), binding.MK_ERR_INVALID_ARG),
+    (dict(scale=float("nan")), binding.MK_ERR_INVALID_ARG),
+    (dict(D=96), binding.MK_ERR_UNSUPPORTED),
+    (dict(Hq=65536 * 2, Hkv=2), binding.MK_ERR_UNSUPPORTED),
+    (dict(workspace_bytes=2 * 8 * 256 * 4 - 4), binding.MK_ERR_INVALID_ARG),
+    (dict(dq=7 * A + 8), binding.MK_ERR_ALIGNMENT),
+    (dict(workspace=10 * A + 4), binding.MK_ERR_ALIGNMENT),
+    (dict(lse=5 * A + 2), binding.MK_ERR_ALIGNMENT),
+])
+def test_backward_rejects_on_host(lib, kw, want):
+    args = dict(BWD_GOOD)
+    args.update(kw)
+    assert binding.mk_attn_bwd_stages(**args) == want
+
+
+DEC_GOOD = dict(q=A, k_cache=2 * A, v_cache=3 * A, page_table=4 * A, seq_lens=5 * A, o=6 * A,
+                lse=7 * A, B=4, Hq=8, Hkv=2, D=128, page_size=64, max_pages=16, num_pages=64,
+                scale=0.088, workspace=None, workspace_bytes=0, stream=None)
+
+
+@pytest.mark.parametrize("kw, want", [
+    (dict(q=None), binding.MK_ERR_INVALID_ARG),
+    (dict(page_table=None), binding.MK_ERR_INVALID_ARG),
+    (dict(Hkv=3), binding.MK_ERR_INVALID_ARG),
+    (dict(max_pages=0), binding.MK_ERR_INVALID_ARG),
+    (dict(scale=float("inf")), binding.MK_ERR_INVALID_ARG),
+    (dict(D=256), binding.MK_ERR_UNSUPPORTED),
+    (dict(page_size=48), binding.MK_ERR_UNSUPPORTED),
+    (dict(B=70000), binding.MK_ERR_UNSUPPORTED),
+    (dict(num_pages=1 << 26), binding.MK_ERR_INVALID_ARG),
+    (dict(o=6 * A + 8), binding.MK_ERR_ALIGNMENT),
+    (dict(seq_lens=5 * A + 2), binding.MK_ERR_ALIGNMENT),
+])
+def test_paged_decode_rejects_on_host(lib, kw, want):
+    args = dict(DEC_GOOD)
+    args.update(kw)
+    assert binding.mk_attn_decode_paged(**args) == want
+
+
+MLA_GOOD = dict(q=A, cache=2 * A, page_table=3 * A, seq_lens=4 * A, o=5 * A, lse=6 * A, B=4,
+                Hq=128, page_size=64, max_pages=16, num_pages=64, scale=0.04, workspace=None,
+                workspace_bytes=0, stream=None)
+
+
+@pytest.mark.parametrize("kw, want", [
+    (dict(cache=None), binding.MK_ERR_INVALID_ARG),
+    (dict(B=0), binding.MK_ERR_INVALID_ARG),
+    (dict(num_pages=0), binding.MK_ERR_INVALID_ARG),
+    (dict(scale=float("nan")), binding.MK_ERR_INVALID_ARG),
+    (dict(page_size=8), binding.MK_ERR_UNSUPPORTED),
+    (dict(max_pages=1 << 26), binding.MK_ERR_INVALID_ARG),
+    (dict(q=A + 8), binding.MK_ERR_ALIGNMENT),
+    (dict(lse=6 * A + 2), binding.MK_ERR_ALIGNMENT),
+])
+def test_latent_decode_rejects_on_host(lib, kw, want):
+    args = dict(MLA_GOOD)
+    args.update(kw)
+    assert binding.mk_attn_mla_decode_paged(**args) == want
