@@ -74,3 +74,13 @@ def test_sample_rows_cover_last_tiles():
         got = {int(i) for (bb, h, i) in rows if bb == b}
         assert set(range(last0, L)) <= got
         assert all(0 <= i < L for (bb, h, i) in rows if bb == b)
+
+
+def test_many_short_lengths():
+    """Seeded, 0..39 with empty sequences among them, 300 at n - 50 and 129 last."""
+    a = W.many_short_lengths(2100, seed=91)
+    assert a == W.many_short_lengths(2100, seed=91)
+    assert len(a) == 2100 and a[2050] == 300 and a[-1] == 129
+    rest = [x for i, x in enumerate(a) if i not in (2050, 2099)]
+    assert min(rest) == 0 and max(rest) <= 39
+    assert W.many_short_lengths(2100, seed=92) != a
