@@ -247,14 +247,17 @@ def attn_bytes(T: int, Hq: int, Hkv: int, D: int) -> int:
 
 def sample_rows(lengths, Hq: int, n: int, seed: int, tile: int = TILE) -> np.ndarray:
     """A deterministic row sample (b, h, i) for checks at full size: every row
-    of the last query tile of one head per sequence, the first row of every
-    sequence, plus uniform random rows, `n` in total at least."""
+    of the last query tile of every head of every sequence (the rows that see
+    the most keys), the first row of every sequence, plus uniform random rows,
+    `n` in total at least."""
     rng = np.random.default_rng(seed)
     rows = []
     for b, L in enumerate(lengths):
-        h = int(rng.integers(0, Hq))
+        if L <= 0:
+            continue
         last0 = ((L - 1) // tile) * tile
-        rows += [(b, h, i) for i in range(last0, L)]
+        for h in range(Hq):
+            rows += [(b, h, i) for i in range(last0, L)]
         rows.append((b, int(rng.integers(0, Hq)), 0))
     total = sum(lengths)
     cum = np.cumsum([0] + list(lengths))

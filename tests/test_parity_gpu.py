@@ -237,13 +237,20 @@ def test_adversarial_rows():
 
 
 def test_large_logits_do_not_overflow():
+    """sigma = 4 and scale 1: logits reach the hundreds and rows are nearly
+    one-hot, while |o| reaches about 16, where one bf16 ulp is 0.125.  The
+    element bound is therefore taken relative to max |o_ref| (1e-2 of it, the
+    2e-2 of unit-scale outputs at |o| <= 2); the relative RMS bound is the
+    usual one, and the lse bound grows with |lse| (fp32)."""
     q, k, v, _ = W.make_qkv(1, 2, 2, 384, 128, seed=404, sigma=4.0)
     o, lse = gpu_attn(q, k, v, True, 1.0)
     o_ref, lse_ref = oracle.attn_fwd(q, k, v, True, 1.0)
     max_abs, rel_rms, lse_err = errors(o, lse, o_ref, lse_ref)
-    # logits up to ~hundreds: the softmax is nearly one-hot, so bf16 P rounding
-    # still bounds the error; lse error scales with |lse| (fp32).
-    assert max_abs <= 5e-2 and lse_err <= 1e-4 * float(np.max(np.abs(lse_ref))) + 1e-3
+    o_scale = float(np.max(np.abs(o_ref)))
+    assert o_scale > 4.0  # the case really has large outputs
+    assert max_abs <= 1e-2 * o_scale, f"max_abs {max_abs:.3e} vs max|o_ref| {o_scale:.3e}"
+    assert rel_rms <= O_REL_RMS, f"rel_rms {rel_rms:.3e}"
+    assert lse_err <= 1e-4 * float(np.max(np.abs(lse_ref))) + 1e-3
 
 
 # --------------------------------------------------------------- invariants
@@ -341,6 +348,11 @@ def _config_parity(n, full: bool, n_rows: int = 4096):
         assert_close(o, lse, o_ref, lse_ref, c.name)
         return
     rows = W.sample_rows(inp.lengths, c.Hq, n_rows, seed=c.seed)
+    # every row of the last query tile of every head is in the sample
+    for b, L in enumerate(inp.lengths):
+        last0 = ((L - 1) // W.TILE) * W.TILE
+        in_last = rows[(rows[:, 0] == b) & (rows[:, 2] >= last0)]
+        assert len({(int(h), int(i)) for _, h, i in in_last}) == c.Hq * (L - last0)
     o_ref, lse_ref = oracle.attn_rows(inp.q, inp.k, inp.v, c.causal, c.scale, rows,
                                       cu_seqlens=None if cu is None else cu.numpy())
     og = np.empty_like(o_ref)
@@ -367,15 +379,19 @@ def test_config2_full():
 
 
 def test_config3_sampled_rows():
-    _config_parity(3, full=False)
+    """S = 32768 (about 8.8 TFLOP in fp64, minutes of host time): the last
+    query tile of all 32 heads (4096 rows that see 32641-32768 keys each),
+    the first row, and 4095 uniform random rows."""
+    _config_parity(3, full=False, n_rows=8192)
 
 
 def test_config4_full():
     _config_parity(4, full=True)
 
 
-def test_config5_sampled_rows():
-    _config_parity(5, full=False)
+def test_config5_full():
+    """Every row of the varlen workload (about 1.5 TFLOP in fp64)."""
+    _config_parity(5, full=True)
 
 
 def test_varlen_causal_beyond_schedule_table():
