@@ -4,9 +4,13 @@
 
 A step is one call of the whole hot path -- mk_attn_fwd, one kernel launch --
 on one batch of seeded synthetic input already resident in HBM.  The default
-workload is the causal GQA forward B=4, Hq=32, Hkv=8, S=2048, D=128 (config
-2); --config selects another of the five.  L2 is flushed (a 256 MiB device
-write) before every timed step, outside the step's CUDA-event pair.
+workload is the largest of the five configurations, the causal GQA
+long-context forward B=1, Hq=32, Hkv=8, S=32768, D=128 (config 3); --config
+selects another.  L2 is flushed (a 256 MiB device write) before every timed
+step, outside the step's CUDA-event pair.  Before the warm-up steps, the step
+runs back to back, untimed, for --settle-s seconds, so that the clocks under
+this load have settled (and are sampled over seconds) when the timed region
+starts.
 
 Under torchrun (N > 1) every rank runs an independent replica of the workload
 on its own GPU (weak scaling: the work units of attention -- sequence, head,
@@ -67,7 +71,11 @@ def parse_args():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5])
+    ap.add_argument("--config", type=int, default=None, choices=[1, 2, 3, 4, 5],
+                    help="workload configuration; default 3 (the largest) for prefill, "
+                         "2 for backward")
+    ap.add_argument("--settle-s", type=float, default=2.5,
+                    help="seconds of untimed back-to-back steps before the warm-up")
     ap.add_argument("--workload", default="prefill",
                     choices=["prefill", "decode", "backward", "mla"],
                     help="prefill: the attention forward pass (--config); decode: one paged "
@@ -76,7 +84,10 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="target CPU time of the oracle baseline sample")
-    return ap.parse_args()
+    args = ap.parse_args()
+    if args.config is None:
+        args.config = 2 if args.workload == "backward" else 3
+    return args
 
 
 # ------------------------------------------------------------------ helpers
@@ -237,20 +248,23 @@ def cpu_oracle_sample(inp, seconds: float, seed: int):
         n_keys = (rows[:, 2] + 1) if c.causal else np.array([inp.lengths[b] for b in rows[:, 0]])
         return float(np.sum(n_keys)) * 4.0 * c.D
 
-    calib = W.sample_rows(inp.lengths, c.Hq, 4 * cores, seed=c.seed + 1)[-4 * cores:]
+    total_rows = sum(inp.lengths) * c.Hq
+    starts = np.cumsum([0] + list(inp.lengths))
+
+    def uniform_rows(rng, n):
+        pick = np.sort(rng.choice(total_rows, size=n, replace=False))  # (token, head) pairs
+        tok, head = pick // c.Hq, pick % c.Hq
+        b = np.searchsorted(starts, tok, side="right") - 1
+        return np.stack([b, head, tok - starts[b]], axis=1).astype(np.int64)
+
+    calib = uniform_rows(np.random.default_rng(c.seed + 1), min(total_rows, 4 * cores))
     t0 = time.perf_counter()
     oracle.attn_rows(inp.q, inp.k, inp.v, c.causal, c.scale, calib, cu_seqlens=cu)
     rate = flops_of(calib) / max(time.perf_counter() - t0, 1e-6)
-    rng = np.random.default_rng(c.seed + 2)
-    total_rows = sum(inp.lengths) * c.Hq
     per_row = 4.0 * c.D * (sum(L * (L + 1) / 2 for L in inp.lengths) if c.causal
                            else sum(L * L for L in inp.lengths)) / sum(inp.lengths)
     n = int(min(total_rows, max(cores, seconds * rate / per_row)))
-    starts = np.cumsum([0] + list(inp.lengths))
-    pick = np.sort(rng.choice(total_rows, size=n, replace=False))  # (token, head) pairs
-    tok, head = pick // c.Hq, pick % c.Hq
-    b = np.searchsorted(starts, tok, side="right") - 1
-    rows = np.stack([b, head, tok - starts[b]], axis=1).astype(np.int64)
+    rows = uniform_rows(np.random.default_rng(c.seed + 2), n)
     t0 = time.perf_counter()
     o, lse = oracle.attn_rows(inp.q, inp.k, inp.v, c.causal, c.scale, rows, cu_seqlens=cu)
     dt = time.perf_counter() - t0
@@ -263,6 +277,32 @@ def cpu_oracle_sample(inp, seconds: float, seed: int):
 
 
 # ------------------------------------------------------------------ our arm
+
+def settle(step, seconds: float, dev) -> int:
+    """Runs `step` back to back, untimed, for about `seconds` of wall time
+    (synchronising every few launches), so that the GPU reaches the clocks
+    and power it holds under this load before anything is timed.  Returns the
+    number of steps run."""
+    import torch
+    if seconds <= 0:
+        return 0
+    n = 0
+    t_end = time.perf_counter() + seconds
+    while time.perf_counter() < t_end:
+        for _ in range(4):
+            step()
+        n += 4
+        torch.cuda.synchronize(dev)
+    return n
+
+
+def clock_normalised(ms_per_step: float, clocks):
+    """ms per step times the median SM clock under load (MHz): kilocycles per
+    step, comparable across runs at different clocks."""
+    if not clocks or not clocks.get("sm_mhz"):
+        return None
+    return round(ms_per_step * clocks["sm_mhz"], 2)
+
 
 def max_over_ranks(value: float, world: int, device) -> float:
     """The maximum of `value` over all ranks: the slowest replica sets the job
@@ -368,6 +408,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
     def step():
         attn_fwd(q, k, v, c.causal, c.scale, cu, out=o, lse=lse, stream=stream)
 
+    settle_steps = settle(step, args.settle_s, dev)
     for _ in range(args.warmup):
         flush.zero_()
         step()
@@ -485,6 +526,9 @@ def run_ours(args, rank: int, world: int, local_rank: int):
             "pct_of_nominal_2250_tflops": round(100.0 * per_launch_tflops / NOMINAL_BF16_TFLOPS, 2),
             "l2": "flushed before every timed step (256 MiB device write, outside the event pair)",
             "timing": "CUDA events around each launch on the launching stream; sum over steps",
+            "settle": f"{settle_steps} untimed back-to-back steps ({args.settle_s} s) before the "
+                      f"{args.warmup} warm-up steps",
+            "ms_per_step_x_sm_mhz": clock_normalised(ms_per_step, clocks),
             "parallelism": f"replicas x{world} (independent workloads per GPU)",
         },
         "roofline": {
@@ -495,7 +539,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
             "frac": round(per_launch_tflops / peak, 4),
             "traffic": ncu_traffic(c.name),
             "peak_source": f"{peak_src} bf16 burst (MEASURED_PEAKS.json bf16_tflops)",
-            "kernel": f"mk::fmha_fwd_kernel<{c.D}>",
+            "kernel": f"mk::mk_attn_fwd_persistent<{c.D}, {int(c.varlen)}>",
         },
         "e2e": {"value": round(e2e_tflops, 2), "unit": "TFLOP/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "mode": E2E_PIPELINED,

@@ -42,9 +42,31 @@ typedef enum {
     MK_ERR_ALIGNMENT = -3,    /* a base pointer not 16-byte aligned */
     MK_ERR_CUDA = -4,         /* a CUDA runtime/driver call failed */
     MK_ERR_TIMEOUT = -5,      /* a kernel wait ran out; reported by mk_attn_check_status */
-    MK_ERR_SCRATCH_LIMIT = -6 /* sizes need more than MK_ATTN_DECODE_STATIC_SCRATCH_BYTES of
-                                 scratch (mk_attn_decode_paged_noalloc only) */
+    MK_ERR_SCRATCH_LIMIT = -6, /* sizes need more than MK_ATTN_DECODE_STATIC_SCRATCH_BYTES of
+                                  scratch (mk_attn_decode_paged_noalloc only) */
+    MK_ERR_BOUNDS = -7         /* a kernel's store index fell outside its output; checked
+                                  only by the check build (MK_DEBUG), reported by
+                                  mk_attn_check_status */
 } mk_status;
+
+/*
+ * Check mode and check build.
+ *
+ *   MK_ATTN_DEBUG  environment variable, read once at the first call.  Set
+ *                  to a nonzero value, every entry point that enqueued work
+ *                  synchronises its stream before returning and returns what
+ *                  mk_attn_check_status reports (MK_OK, MK_ERR_TIMEOUT,
+ *                  MK_ERR_INVALID_ARG, MK_ERR_BOUNDS, MK_ERR_CUDA) instead of
+ *                  MK_OK: a device-side error is then tied to the call that
+ *                  caused it.  Such calls are no longer asynchronous.
+ *   MK_DEBUG       compile definition of the check build of this library
+ *                  (libmk_attn_debug.so).  Every kernel then checks the index
+ *                  of each global-memory store of its outputs, partials and
+ *                  workspace against the sizes of the call; an index out of
+ *                  range skips the store and records MK_ERR_BOUNDS for
+ *                  mk_attn_check_status.  Nothing traps.  The release build
+ *                  carries none of these checks.
+ */
 
 /*
  * mk_attn_fwd -- attention forward pass (causal or not, GQA, optional varlen).
@@ -222,8 +244,14 @@ MK_API int mk_attn_decode_paged(const void *q, const void *k_cache, const void *
                                 int max_pages, int num_pages, float scale, void *workspace,
                                 int64_t workspace_bytes, void *stream);
 
-/* Size of the library's own decode scratch array (16 MiB), which every GPU
- * that loads the library holds until the process exits. */
+/* Size of the library's own decode scratch array (16 MiB).  It belongs to
+ * the code of the paged decode step, and a GPU reserves it when that code is
+ * loaded on it: at the first decode call on the device (either decode entry
+ * point), or at context creation when the CUDA runtime loads modules eagerly
+ * (CUDA_MODULE_LOADING=EAGER).  It stays reserved until the process exits.
+ * Callers that never run a decode step do not load that code and do not
+ * hold the array (mk_attn_check_status reads only the status words of the
+ * kernel families that have run on the device). */
 #define MK_ATTN_DECODE_STATIC_SCRATCH_BYTES (16 * 1024 * 1024)
 
 /*
@@ -237,13 +265,22 @@ MK_API int mk_attn_decode_paged(const void *q, const void *k_cache, const void *
  * without `workspace` and `workspace_bytes`: the per-split partial results
  * go to a scratch array of MK_ATTN_DECODE_STATIC_SCRATCH_BYTES bytes that
  * the library declares in device memory (one per GPU).  The call allocates
- * nothing and calls no allocating routine.
+ * nothing and calls no allocating routine; the array itself is reserved when
+ * the decode code loads on the device (see MK_ATTN_DECODE_STATIC_SCRATCH_BYTES),
+ * which the first call does if nothing loaded it before.  A caller whose
+ * device memory another allocator will take should therefore make one call
+ * at start-up, before that allocator claims the device: if the device has no
+ * room left for the array when the code loads, that call returns MK_ERR_CUDA.
  *
- *   - Sizes for which mk_attn_decode_workspace_bytes() exceeds
+ *   - Checks run in this order, and the first that fails decides the
+ *     status: the host argument checks of mk_attn_decode_paged (no CUDA
+ *     call); then the scratch size: sizes for which
+ *     mk_attn_decode_workspace_bytes() exceeds
  *     MK_ATTN_DECODE_STATIC_SCRATCH_BYTES return MK_ERR_SCRATCH_LIMIT and
- *     launch nothing; use mk_attn_decode_paged with a workspace for those.
- *   - The first call on each device looks up that device's address of the
- *     array (with the device current) and keeps it; make that first call
+ *     launch nothing (use mk_attn_decode_paged with a workspace for those);
+ *     then the array's address.
+ *   - The first valid call on each device looks up that device's address of
+ *     the array (with the device current) and keeps it; make that first call
  *     before any stream capture on the device.  A failed lookup returns
  *     MK_ERR_CUDA.
  *   - Every call on a device shares the one array, which keeps whatever the
@@ -366,11 +403,13 @@ MK_API const char *mk_attn_error_string(int status);
 
 /*
  * mk_attn_check_status -- synchronises `stream`, then reads and clears the
- * device status words written by kernels (forward, backward, decode) whose
- * internal waits ran out or that met device-side inputs out of range (decode
- * page tables, lengths).
- * Returns MK_OK, MK_ERR_TIMEOUT, MK_ERR_INVALID_ARG, or MK_ERR_CUDA if
- * synchronisation failed.
+ * device status words written by kernels (forward, backward, decode, latent
+ * decode) whose internal waits ran out, that met device-side inputs out of
+ * range (decode page tables, lengths), or (check build only) whose store
+ * index checks failed.  Only the families that have enqueued a kernel on the
+ * current device are read, so the call loads no kernel code of its own.
+ * Returns MK_OK, MK_ERR_TIMEOUT, MK_ERR_INVALID_ARG, MK_ERR_BOUNDS, or
+ * MK_ERR_CUDA if synchronisation failed.
  */
 MK_API int mk_attn_check_status(void *stream);
 

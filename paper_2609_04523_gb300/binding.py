@@ -11,7 +11,13 @@ import os
 import threading
 
 PKG = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(PKG, "libmk_attn.so")
+RELEASE_LIB_PATH = os.path.join(PKG, "libmk_attn.so")
+CHECK_LIB_PATH = os.path.join(PKG, "libmk_attn_debug.so")
+# MK_ATTN_CHECK_BUILD=1 in the environment loads the check build (compiled
+# with MK_DEBUG: store indices checked in every kernel) instead of the release
+# build.  Build it with paper_2609_04523_gb300.build.build_library(debug=True).
+LIB_PATH = (CHECK_LIB_PATH if os.environ.get("MK_ATTN_CHECK_BUILD", "0") not in ("", "0")
+            else RELEASE_LIB_PATH)
 
 MK_OK = 0
 MK_ERR_INVALID_ARG = -1
@@ -20,6 +26,7 @@ MK_ERR_ALIGNMENT = -3
 MK_ERR_CUDA = -4
 MK_ERR_TIMEOUT = -5
 MK_ERR_SCRATCH_LIMIT = -6
+MK_ERR_BOUNDS = -7
 
 # Backward-pass stages (MK_BWD_* in include/mk_attn.h).
 BWD_DELTA, BWD_DKDV, BWD_DQ, BWD_ALL = 1, 2, 4, 7

@@ -413,6 +413,11 @@ __global__ void __launch_bounds__(kThreads, MH > 4 ? 2 : 3)
       const float inv_l = lt > 0.f ? 1.f / lt : 0.f;
       const float lse = lt > 0.f ? (M + log2f(lt)) * 0.69314718055994530942f : -INFINITY;
       const int hq = h0 + h;
+      // Check build: the (sequence, head) row and the split lie inside the
+      // outputs and the partials.
+      if (!dbg_in_range((int64_t)b * p.Hq + hq, (int64_t)p.B * p.Hq, &g_status) ||
+          !dbg_in_range(split, p.n_splits, &g_status))
+        continue;
       if (p.n_splits == 1) {
         uint16_t *orow = p.o + ((int64_t)b * p.Hq + hq) * D + lane * (D / 32);
 #pragma unroll
@@ -548,6 +553,7 @@ static int launch(const CUtensorMap &tk, const CUtensorMap &tv, const Params &p,
                            (int)sm) != cudaSuccess)
     return MK_ERR_CUDA;
   const dim3 grid(p.n_splits, p.Hkv * p.head_groups, p.B);
+  mark_launched(kFamDecode);
   decode_kernel<D, MH><<<grid, kThreads, sm, st>>>(tk, tv, p);
   if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
   if (p.n_splits > 1) {
@@ -588,9 +594,41 @@ static void *static_scratch_address() {
   return g_scratch.addr[dev];
 }
 
+// The checks of mk_attn_decode_paged that need neither the device nor the
+// workspace: pointers, sizes, head dimension, page size, grid limits and
+// alignment.  No CUDA call; shared by both decode entry points so that they
+// reject the same arguments with the same status.
+static int check_host_args(const void *q, const void *k_cache, const void *v_cache,
+                           const int32_t *page_table, const int32_t *seq_lens, const void *o,
+                           const float *lse, int B, int Hq, int Hkv, int D, int page_size,
+                           int max_pages, int num_pages, float scale) {
+  if (!q || !k_cache || !v_cache || !page_table || !seq_lens || !o || !lse)
+    return MK_ERR_INVALID_ARG;
+  if (B < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || max_pages < 1 || num_pages < 1)
+    return MK_ERR_INVALID_ARG;
+  if (!std::isfinite(scale)) return MK_ERR_INVALID_ARG;
+  if (D != 64 && D != 128) return MK_ERR_UNSUPPORTED;
+  if (page_size != 16 && page_size != 32 && page_size != 64 && page_size != 128)
+    return MK_ERR_UNSUPPORTED;
+  int HG = 1, head_groups = 1;
+  head_split(Hq / Hkv, HG, head_groups);
+  if (B > 65535 || (int64_t)Hkv * head_groups > 65535) return MK_ERR_UNSUPPORTED;  // grid z / y
+  if ((int64_t)num_pages * page_size > INT32_MAX || (int64_t)max_pages * page_size > INT32_MAX)
+    return MK_ERR_INVALID_ARG;
+  auto misaligned = [](const void *ptr, uintptr_t a) {
+    return (reinterpret_cast<uintptr_t>(ptr) & (a - 1)) != 0;
+  };
+  if (misaligned(q, 16) || misaligned(k_cache, 16) || misaligned(v_cache, 16) ||
+      misaligned(o, 16) || misaligned(lse, 4) || misaligned(page_table, 4) ||
+      misaligned(seq_lens, 4))
+    return MK_ERR_ALIGNMENT;
+  return MK_OK;
+}
+
 }  // namespace dec
 
 int decode_take_status() {
+  if (!launched(kFamDecode)) return 0;
   int h = 0;
   if (cudaMemcpyFromSymbol(&h, dec::g_status, sizeof(int)) != cudaSuccess) return MK_ERR_CUDA;
   if (h != 0) {
@@ -618,31 +656,21 @@ int64_t mk_attn_decode_workspace_bytes(int B, int Hq, int Hkv, int D, int page_s
   return (int64_t)B * Hq * n_splits * (D + 1) * 4;
 }
 
-int mk_attn_decode_paged(const void *q, const void *k_cache, const void *v_cache,
-                         const int32_t *page_table, const int32_t *seq_lens, void *o, float *lse,
-                         int B, int Hq, int Hkv, int D, int page_size, int max_pages,
-                         int num_pages, float scale, void *workspace, int64_t workspace_bytes,
-                         void *stream) {
-  using namespace mk;
-  if (!q || !k_cache || !v_cache || !page_table || !seq_lens || !o || !lse)
-    return MK_ERR_INVALID_ARG;
-  if (B < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv != 0 || max_pages < 1 || num_pages < 1)
-    return MK_ERR_INVALID_ARG;
+}  // extern "C"
 
-  if (!std::isfinite(scale)) return MK_ERR_INVALID_ARG;
-  if (D != 64 && D != 128) return MK_ERR_UNSUPPORTED;
-  if (page_size != 16 && page_size != 32 && page_size != 64 && page_size != 128)
-    return MK_ERR_UNSUPPORTED;
+namespace mk {
+static int decode_paged_impl(const void *q, const void *k_cache, const void *v_cache,
+                             const int32_t *page_table, const int32_t *seq_lens, void *o,
+                             float *lse, int B, int Hq, int Hkv, int D, int page_size,
+                             int max_pages, int num_pages, float scale, void *workspace,
+                             int64_t workspace_bytes, void *stream) {
+  const int chk = dec::check_host_args(q, k_cache, v_cache, page_table, seq_lens, o, lse, B, Hq,
+                                       Hkv, D, page_size, max_pages, num_pages, scale);
+  if (chk != MK_OK) return chk;
+  auto misaligned = [](const void *ptr, uintptr_t a) { return (reinterpret_cast<uintptr_t>(ptr) & (a - 1)) != 0; };
   const int G = Hq / Hkv;
   int HG = 1, head_groups = 1;
   dec::head_split(G, HG, head_groups);
-  if (B > 65535 || (int64_t)Hkv * head_groups > 65535) return MK_ERR_UNSUPPORTED;  // grid z / y
-  if ((int64_t)num_pages * page_size > INT32_MAX || (int64_t)max_pages * page_size > INT32_MAX)
-    return MK_ERR_INVALID_ARG;
-  auto misaligned = [](const void *ptr, uintptr_t a) { return (reinterpret_cast<uintptr_t>(ptr) & (a - 1)) != 0; };
-  if (misaligned(q, 16) || misaligned(k_cache, 16) || misaligned(v_cache, 16) || misaligned(o, 16) ||
-      misaligned(lse, 4) || misaligned(page_table, 4) || misaligned(seq_lens, 4))
-    return MK_ERR_ALIGNMENT;
   const int sms = dec::sm_count();
   if (sms <= 0) return MK_ERR_CUDA;
   dec::Params p;
@@ -686,22 +714,45 @@ int mk_attn_decode_paged(const void *q, const void *k_cache, const void *v_cache
   if (HG <= 4) return dec::launch<64, 4>(tk, tv, p, st);
   return dec::launch<64, dec::kMaxHeads>(tk, tv, p, st);
 }
+}  // namespace mk
+
+extern "C" {
+
+int mk_attn_decode_paged(const void *q, const void *k_cache, const void *v_cache,
+                         const int32_t *page_table, const int32_t *seq_lens, void *o, float *lse,
+                         int B, int Hq, int Hkv, int D, int page_size, int max_pages,
+                         int num_pages, float scale, void *workspace, int64_t workspace_bytes,
+                         void *stream) {
+  return mk::finish_call(mk::decode_paged_impl(q, k_cache, v_cache, page_table, seq_lens, o, lse,
+                                               B, Hq, Hkv, D, page_size, max_pages, num_pages,
+                                               scale, workspace, workspace_bytes, stream),
+                         stream);
+}
 
 
 int mk_attn_decode_paged_noalloc(const void *q, const void *k_cache, const void *v_cache,
                                  const int32_t *page_table, const int32_t *seq_lens, void *o,
                                  float *lse, int B, int Hq, int Hkv, int D, int page_size,
                                  int max_pages, int num_pages, float scale, void *stream) {
-  // Set-up on the first call per device, whether or not these sizes need
-  // scratch, so that the lookup never happens later during a stream capture.
+  // Host checks first (no CUDA call), then the scratch size, then the
+  // once-per-device address lookup; so an invalid call returns the status
+  // mk_attn_decode_paged gives it and touches nothing on the device.
+  const int chk = mk::dec::check_host_args(q, k_cache, v_cache, page_table, seq_lens, o, lse, B,
+                                           Hq, Hkv, D, page_size, max_pages, num_pages, scale);
+  if (chk != MK_OK) return chk;
+  const int64_t need = mk_attn_decode_workspace_bytes(B, Hq, Hkv, D, page_size, max_pages);
+  if (need < 0) return MK_ERR_CUDA;  // valid sizes: only the device query can fail
+  if (need > mk::dec::kStaticScratchBytes) return MK_ERR_SCRATCH_LIMIT;
+  // The lookup happens on the first valid call per device, whether or not
+  // these sizes need scratch, so that it never happens later during a stream
+  // capture.
   void *scratch = mk::dec::static_scratch_address();
   if (!scratch) return MK_ERR_CUDA;
-  const int64_t need = mk_attn_decode_workspace_bytes(B, Hq, Hkv, D, page_size, max_pages);
-  if (need > mk::dec::kStaticScratchBytes) return MK_ERR_SCRATCH_LIMIT;
-  // Invalid sizes (need < 0) are reported by the checks of mk_attn_decode_paged.
-  return mk_attn_decode_paged(q, k_cache, v_cache, page_table, seq_lens, o, lse, B, Hq, Hkv, D,
-                              page_size, max_pages, num_pages, scale, scratch,
-                              mk::dec::kStaticScratchBytes, stream);
+  return mk::finish_call(
+      mk::decode_paged_impl(q, k_cache, v_cache, page_table, seq_lens, o, lse, B, Hq, Hkv, D,
+                            page_size, max_pages, num_pages, scale, scratch,
+                            mk::dec::kStaticScratchBytes, stream),
+      stream);
 }
 
 }  // extern "C"

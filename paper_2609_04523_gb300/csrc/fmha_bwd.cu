@@ -657,7 +657,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             // Every elementwise thread has read the dO tile: release it.
             if (threadIdx.x == 0) mbar_arrive(&ctl->fixed_empty);
             row_dl = vec[row] + vec[kTile + row];
-            if (wg == 0 && qpos < w.len) p.delta[ri] = row_dl;
+            if (wg == 0 && qpos < w.len &&
+                dbg_in_range(ri, (int64_t)p.Hq * (p.varlen ? p.S : (int64_t)p.B * p.S),
+                             &g_status))
+              p.delta[ri] = row_dl;
           }
         } else {
           // The producer lanes wrote this slot's vectors before arriving on
@@ -743,8 +746,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
       tc_fence_after_sync();
       const int pos = w.tile * kTile + row;
-      const bool valid = pos < w.len;
       const int64_t tok = (int64_t)w.seq_start + pos;
+      // Check build: the row lies inside its output (tokens x heads rows).
+      const bool valid = pos < w.len &&
+                         dbg_in_range(tok, p.varlen ? (int64_t)p.S : (int64_t)p.B * p.S,
+                                      &g_status) &&
+                         dbg_in_range(w.head, DQ ? p.Hq : p.Hkv, &g_status);
       // This warpgroup stores columns wg * D/2 .. + D/2 of its row.
       auto store_acc = [&](uint32_t col, uint16_t *base, int heads, int head, float mul) {
         uint4 *dst = reinterpret_cast<uint4 *>(base + (tok * heads + head) * (int64_t)D + wg * (D / 2));
@@ -861,6 +868,7 @@ static int launch(const void *q, const void *k, const void *v, const void *o, co
   const int v0 = D == 128 ? 2 : 0;
   if (di.sm_count <= 0 || di.attr_err[v0] != cudaSuccess || di.attr_err[v0 + 1] != cudaSuccess)
     return MK_ERR_CUDA;
+  mark_launched(kFamBwd);
   // The dQ kernel computes Delta for its own rows; the separate Delta kernel
   // runs only when Delta is asked for without dQ.
   if ((stages & MK_BWD_DELTA) && !(stages & MK_BWD_DQ)) {
@@ -895,6 +903,7 @@ static int launch(const void *q, const void *k, const void *v, const void *o, co
 }  // namespace bwd
 
 int bwd_take_status() {
+  if (!launched(kFamBwd)) return 0;
   int h = 0;
   if (cudaMemcpyFromSymbol(&h, bwd::g_status, sizeof(int)) != cudaSuccess) return MK_ERR_CUDA;
   if (h != 0) {
@@ -914,12 +923,14 @@ int64_t mk_attn_bwd_workspace_bytes(int B, int Hq, int S, int varlen) {
   return rows * 4;
 }
 
-int mk_attn_bwd_stages(const void *q, const void *k, const void *v, const void *o,
-                       const float *lse, const void *dO, void *dq, void *dk, void *dv, int B,
-                       int Hq, int Hkv, int S, int D, int causal, float scale,
-                       const int32_t *cu_seqlens, void *workspace, int64_t workspace_bytes,
-                       int stages, void *stream) {
-  using namespace mk;
+}  // extern "C"
+
+namespace mk {
+static int attn_bwd_impl(const void *q, const void *k, const void *v, const void *o,
+                         const float *lse, const void *dO, void *dq, void *dk, void *dv, int B,
+                         int Hq, int Hkv, int S, int D, int causal, float scale,
+                         const int32_t *cu_seqlens, void *workspace, int64_t workspace_bytes,
+                         int stages, void *stream) {
   if (stages < 1 || stages > MK_BWD_ALL) return MK_ERR_INVALID_ARG;
   if (!q || !k || !v || !o || !lse || !dO || !dq || !dk || !dv || !workspace)
     return MK_ERR_INVALID_ARG;
@@ -964,6 +975,20 @@ int mk_attn_bwd_stages(const void *q, const void *k, const void *v, const void *
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (D == 128) return bwd::launch<128>(q, k, v, o, dO, p, tokens, stages, st);
   return bwd::launch<64>(q, k, v, o, dO, p, tokens, stages, st);
+}
+}  // namespace mk
+
+extern "C" {
+
+int mk_attn_bwd_stages(const void *q, const void *k, const void *v, const void *o,
+                       const float *lse, const void *dO, void *dq, void *dk, void *dv, int B,
+                       int Hq, int Hkv, int S, int D, int causal, float scale,
+                       const int32_t *cu_seqlens, void *workspace, int64_t workspace_bytes,
+                       int stages, void *stream) {
+  return mk::finish_call(mk::attn_bwd_impl(q, k, v, o, lse, dO, dq, dk, dv, B, Hq, Hkv, S, D,
+                                           causal, scale, cu_seqlens, workspace,
+                                           workspace_bytes, stages, stream),
+                         stream);
 }
 
 int mk_attn_bwd(const void *q, const void *k, const void *v, const void *o, const float *lse,

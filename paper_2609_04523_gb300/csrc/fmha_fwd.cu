@@ -331,7 +331,7 @@ __device__ __forceinline__ void drain_wait(uint64_t *bar, uint32_t parity) {
 
 template <int D, bool VL>
 __global__ void __launch_bounds__(kThreads, 1)
-    fmha_fwd_kernel(const __grid_constant__ CUtensorMap tm_q,
+    mk_attn_fwd_persistent(const __grid_constant__ CUtensorMap tm_q,
                     const __grid_constant__ CUtensorMap tm_k,
                     const __grid_constant__ CUtensorMap tm_v, const Params p) {
   using C = KernelCfg<D>;
@@ -826,6 +826,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after_sync();
       const float inv_l = 1.f / l_run;
       const int64_t tok = (int64_t)w.seq_start + qpos;
+      // Check build: the row lies inside o and lse (tokens x Hq rows).
+      const bool row_store =
+          row_valid &&
+          dbg_in_range(tok, VL ? (int64_t)p.S : (int64_t)p.B * p.S, &g_status) &&
+          dbg_in_range(w.hq, p.Hq, &g_status);
       uint4 *dst = reinterpret_cast<uint4 *>(p.o + (tok * p.Hq + w.hq) * (int64_t)D);
 #pragma unroll
       for (int c = 0; c < D / 32; ++c) {
@@ -838,7 +843,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int e = 0; e < 16; ++e)
           v[e] = pack_bf16x2(__uint_as_float(o_raw[2 * e]) * inv_l,
                              __uint_as_float(o_raw[2 * e + 1]) * inv_l);
-        if (row_valid) {
+        if (row_store) {
           // Each thread writes its own row: 32-byte stores fill whole sectors
           // (half as many store instructions and sector writes as 16-byte ones).
           if (p.o_align32) {
@@ -856,7 +861,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // O_X has been read: the next unit's first P_X V (which overwrites O_X)
       // is issued only after this warpgroup produces that unit's P_X(0).
       tc_fence_before_sync();
-      if (row_valid) {
+      if (row_store) {
         const float lse = (m_run + log2f(l_run)) * 0.69314718055994530942f;
         const int64_t li = VL ? (int64_t)w.hq * p.S + tok
                                     : ((int64_t)w.b * p.Hq + w.hq) * p.S + qpos;
@@ -896,11 +901,11 @@ static DeviceInfo g_devices[64];
 template <int D, bool VL>
 static void kernel_setup(DeviceInfo &di) {
   const int vi = (D == 128 ? 2 : 0) + (VL ? 1 : 0);
-  di.attr_err[vi] = cudaFuncSetAttribute(fmha_fwd_kernel<D, VL>,
+  di.attr_err[vi] = cudaFuncSetAttribute(mk_attn_fwd_persistent<D, VL>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          KernelCfg<D>::kSmemBytes);
   cudaFuncAttributes fa;
-  if (cudaFuncGetAttributes(&fa, fmha_fwd_kernel<D, VL>) == cudaSuccess) di.regs[vi] = fa.numRegs;
+  if (cudaFuncGetAttributes(&fa, mk_attn_fwd_persistent<D, VL>) == cudaSuccess) di.regs[vi] = fa.numRegs;
 }
 
 template <int D, bool VL>
@@ -932,7 +937,8 @@ static int launch(const void *q, const void *k, const void *v, const Params &p, 
   const mk_attn_tuning tune = current_tuning();
   const int ctas = tune.ctas > 0 ? tune.ctas : di.sm_count;
   const int grid = p.n_units < ctas ? p.n_units : ctas;
-  fmha_fwd_kernel<D, VL><<<grid, kThreads, C::kSmemBytes, stream>>>(tq, tk, tv, p);
+  mark_launched(kFamFwd);
+  mk_attn_fwd_persistent<D, VL><<<grid, kThreads, C::kSmemBytes, stream>>>(tq, tk, tv, p);
   return cudaGetLastError() == cudaSuccess ? MK_OK : MK_ERR_CUDA;
 }
 
@@ -940,6 +946,7 @@ static int launch(const void *q, const void *k, const void *v, const Params &p, 
 
 namespace mk {
 int fwd_take_status() {
+  if (!launched(kFamFwd)) return 0;
   int h = 0;
   if (cudaMemcpyFromSymbol(&h, g_status, sizeof(int)) != cudaSuccess) return MK_ERR_CUDA;
   if (h != 0) {
@@ -1006,13 +1013,17 @@ extern "C" {
 int mk_attn_fwd(const void *q, const void *k, const void *v, void *o, float *lse, int B,
                 int Hq, int Hkv, int S, int D, int causal, float scale,
                 const int32_t *cu_seqlens, void *stream) {
-  return mk::attn_fwd_impl(q, k, v, o, lse, B, Hq, Hkv, S, D, causal, scale, cu_seqlens, stream, 0);
+  return mk::finish_call(
+      mk::attn_fwd_impl(q, k, v, o, lse, B, Hq, Hkv, S, D, causal, scale, cu_seqlens, stream, 0),
+      stream);
 }
 
 int mk_attn_fwd_stall_test(const void *q, const void *k, const void *v, void *o, float *lse,
                            int B, int Hq, int Hkv, int S, int D, int causal, float scale,
                            const int32_t *cu_seqlens, void *stream) {
-  return mk::attn_fwd_impl(q, k, v, o, lse, B, Hq, Hkv, S, D, causal, scale, cu_seqlens, stream, 1);
+  return mk::finish_call(
+      mk::attn_fwd_impl(q, k, v, o, lse, B, Hq, Hkv, S, D, causal, scale, cu_seqlens, stream, 1),
+      stream);
 }
 
 

@@ -403,10 +403,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     const int h = hg * kHeads + row;
     if (ok) {
-      const bool valid = h < p.Hq;
+      const int64_t bh = (int64_t)b * p.Hq + h;
+      // Check build: the (sequence, head) row and the split lie inside the
+      // outputs and the partials.
+      const bool valid = h < p.Hq && dbg_in_range(bh, (int64_t)p.B * p.Hq, &g_status) &&
+                         dbg_in_range(split, p.n_splits, &g_status);
       const float inv_l = l_run > 0.f ? 1.f / l_run : 0.f;
       const float lse = l_run > 0.f ? (m_run + log2f(l_run)) * 0.69314718055994530942f : -INFINITY;
-      const int64_t bh = (int64_t)b * p.Hq + h;
 #pragma unroll 1
       for (int c = 0; c < kDvCta / 32; ++c) {
         float v[32];
@@ -547,6 +550,7 @@ static bool encode(CUtensorMap *map, const void *base, int rank, const cuuint64_
 }  // namespace mla
 
 int mla_take_status() {
+  if (!launched(kFamMla)) return 0;
   int h = 0;
   if (cudaMemcpyFromSymbol(&h, mla::g_status, sizeof(int)) != cudaSuccess) return MK_ERR_CUDA;
   if (h != 0) {
@@ -573,11 +577,13 @@ int64_t mk_attn_mla_decode_workspace_bytes(int B, int Hq, int page_size, int max
   return (int64_t)B * Hq * n_splits * (mk::mla::kDv + 4) * 4;
 }
 
-int mk_attn_mla_decode_paged(const void *q, const void *cache, const int32_t *page_table,
-                             const int32_t *seq_lens, void *o, float *lse, int B, int Hq,
-                             int page_size, int max_pages, int num_pages, float scale,
-                             void *workspace, int64_t workspace_bytes, void *stream) {
-  using namespace mk;
+}  // extern "C"
+
+namespace mk {
+static int mla_decode_impl(const void *q, const void *cache, const int32_t *page_table,
+                           const int32_t *seq_lens, void *o, float *lse, int B, int Hq,
+                           int page_size, int max_pages, int num_pages, float scale,
+                           void *workspace, int64_t workspace_bytes, void *stream) {
   if (!q || !cache || !page_table || !seq_lens || !o || !lse) return MK_ERR_INVALID_ARG;
   if (B < 1 || Hq < 1 || max_pages < 1 || num_pages < 1) return MK_ERR_INVALID_ARG;
   if (!std::isfinite(scale)) return MK_ERR_INVALID_ARG;
@@ -628,6 +634,7 @@ int mk_attn_mla_decode_paged(const void *q, const void *cache, const int32_t *pa
     return MK_ERR_CUDA;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const dim3 grid(2 * B * head_groups, p.n_splits, 1);
+  mark_launched(kFamMla);
   mla::mla_decode_kernel<<<grid, mla::kThreads, mla::kSmemBytes, st>>>(tq, tc, p);
   if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
   if (p.n_splits > 1) {
@@ -635,6 +642,19 @@ int mk_attn_mla_decode_paged(const void *q, const void *cache, const int32_t *pa
     if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
   }
   return MK_OK;
+}
+}  // namespace mk
+
+extern "C" {
+
+int mk_attn_mla_decode_paged(const void *q, const void *cache, const int32_t *page_table,
+                             const int32_t *seq_lens, void *o, float *lse, int B, int Hq,
+                             int page_size, int max_pages, int num_pages, float scale,
+                             void *workspace, int64_t workspace_bytes, void *stream) {
+  return mk::finish_call(mk::mla_decode_impl(q, cache, page_table, seq_lens, o, lse, B, Hq,
+                                             page_size, max_pages, num_pages, scale, workspace,
+                                             workspace_bytes, stream),
+                         stream);
 }
 
 }  // extern "C"

@@ -321,6 +321,23 @@ __device__ __forceinline__ void st_global_v4_hint(void *ptr, uint32_t a0, uint32
                : "memory");
 }
 
+// ------------------------------------------------------------ debug checks
+
+// Bounds check of a global-memory store index, compiled in only when the
+// library is built with MK_DEBUG (the check build): an index outside [0, n)
+// records MK_ERR_BOUNDS in the kernel family's status word (read by
+// mk_attn_check_status) and returns false, so that the caller skips the
+// store.  Never traps.  Without MK_DEBUG it is always true and costs nothing.
+#if defined(MK_DEBUG)
+__device__ __forceinline__ bool dbg_in_range(int64_t i, int64_t n, int *status) {
+  if (i >= 0 && i < n) return true;
+  atomicCAS(status, 0, -7);  // MK_ERR_BOUNDS
+  return false;
+}
+#else
+__device__ __forceinline__ bool dbg_in_range(int64_t, int64_t, int *) { return true; }
+#endif
+
 // ------------------------------------------------------------------ scalars
 
 // 2^x on the MUFU unit (approximate, flush-to-zero; 2^-inf = +0).

@@ -2,6 +2,9 @@
 // the device status check that covers every kernel family, and the version.
 #include <cuda_runtime.h>
 
+#include <atomic>
+#include <cstdlib>
+#include <cstring>
 #include <mutex>
 
 #include "mk_attn.h"
@@ -18,6 +21,33 @@ mk_attn_tuning current_tuning() {
   std::lock_guard<std::mutex> lock(g_tuning_mu);
   return g_tuning;
 }
+
+namespace {
+constexpr int kMaxDevices = 64;
+std::atomic<unsigned> g_launched[kMaxDevices];  // bit f: family f enqueued on device
+}  // namespace
+
+void mark_launched(Family family) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return;
+  g_launched[dev].fetch_or(1u << family, std::memory_order_relaxed);
+}
+
+bool launched(Family family) {
+  int dev = 0;
+  // Unknown device: report "launched" so that the status word is read.
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return true;
+  return (g_launched[dev].load(std::memory_order_relaxed) >> family) & 1u;
+}
+
+int finish_call(int status, void *stream) {
+  static const bool debug = [] {
+    const char *e = std::getenv("MK_ATTN_DEBUG");
+    return e != nullptr && e[0] != '\0' && std::strcmp(e, "0") != 0;
+  }();
+  if (status != MK_OK || !debug) return status;
+  return mk_attn_check_status(stream);
+}
 }  // namespace mk
 
 extern "C" {
@@ -31,6 +61,7 @@ const char *mk_attn_error_string(int status) {
     case MK_ERR_CUDA: return "CUDA call failed";
     case MK_ERR_TIMEOUT: return "kernel wait timed out";
     case MK_ERR_SCRATCH_LIMIT: return "sizes need more scratch than the static decode array holds";
+    case MK_ERR_BOUNDS: return "a store index check of the check build failed";
     default: return "unknown status";
   }
 }

@@ -46,10 +46,24 @@ inline bool encode_tokens_heads_dim(CUtensorMap *map, const void *base, uint64_t
 mk_attn_tuning current_tuning();
 
 // Read and clear the device status word of each kernel family (each defined
-// with its kernels).
+// with its kernels).  A family that has enqueued no kernel on the current
+// device reads as 0 without touching the device, so that a status check never
+// loads the code and device arrays of a family the caller has not used.
 int fwd_take_status();
 int bwd_take_status();
 int decode_take_status();
 int mla_take_status();
+
+enum Family { kFamFwd = 0, kFamBwd = 1, kFamDecode = 2, kFamMla = 3 };
+// Records that `family` enqueues kernels on the current device (called by
+// each launcher before its first launch), and whether it has.
+void mark_launched(Family family);
+bool launched(Family family);
+
+// Check mode: with MK_ATTN_DEBUG set to a nonzero value in the environment
+// (read once, at the first call), every entry point that enqueued work
+// synchronises its stream and returns what mk_attn_check_status reports
+// instead of MK_OK.  Without it, returns `status` unchanged.
+int finish_call(int status, void *stream);
 
 }  // namespace mk

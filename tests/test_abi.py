@@ -162,3 +162,45 @@ def test_latent_decode_rejects_on_host(lib, kw, want):
     args = dict(MLA_GOOD)
     args.update(kw)
     assert binding.mk_attn_mla_decode_paged(**args) == want
+
+
+def test_binding_constants_match_the_header():
+    """Constants the binding restates from include/mk_attn.h."""
+    text = open(os.path.join(ROOT, "include", "mk_attn.h")).read()
+    m = re.search(r"#define\s+MK_ATTN_DECODE_STATIC_SCRATCH_BYTES\s+\(([^)]*)\)", text)
+    assert m, "MK_ATTN_DECODE_STATIC_SCRATCH_BYTES not found"
+    assert eval(m.group(1), {"__builtins__": {}}) == binding.DECODE_STATIC_SCRATCH_BYTES
+    codes = dict(re.findall(r"\b(MK_(?:OK|ERR_\w+))\s*=\s*(-?\d+)", text))
+    assert codes, "status codes not found"
+    for name, val in codes.items():
+        assert getattr(binding, name) == int(val), name
+    for name in ("MK_MLA_DQK", "MK_MLA_DV"):
+        m = re.search(r"#define\s+%s\s+(\d+)" % name, text)
+        assert int(m.group(1)) == getattr(binding, name.replace("MK_", ""))
+
+
+# The allocation-free decode entry point runs the host checks of
+# mk_attn_decode_paged before anything else (no CUDA call), so it rejects the
+# same arguments with the same status.
+@pytest.mark.parametrize("kw, want", [
+    (dict(q=None), binding.MK_ERR_INVALID_ARG),
+    (dict(seq_lens=None), binding.MK_ERR_INVALID_ARG),
+    (dict(Hkv=3), binding.MK_ERR_INVALID_ARG),
+    (dict(num_pages=0), binding.MK_ERR_INVALID_ARG),
+    (dict(scale=float("nan")), binding.MK_ERR_INVALID_ARG),
+    (dict(D=256), binding.MK_ERR_UNSUPPORTED),
+    (dict(page_size=48), binding.MK_ERR_UNSUPPORTED),
+    (dict(page_size=48, B=60000), binding.MK_ERR_UNSUPPORTED),  # not MK_ERR_SCRATCH_LIMIT
+    (dict(B=70000), binding.MK_ERR_UNSUPPORTED),
+    (dict(num_pages=1 << 26), binding.MK_ERR_INVALID_ARG),
+    (dict(o=6 * A + 8), binding.MK_ERR_ALIGNMENT),
+    (dict(lse=7 * A + 2), binding.MK_ERR_ALIGNMENT),
+])
+def test_noalloc_decode_rejects_on_host(lib, kw, want):
+    args = dict(DEC_GOOD)
+    args.update(kw)
+    del args["workspace"], args["workspace_bytes"]
+    assert binding.mk_attn_decode_paged_noalloc(**args) == want
+    full = dict(DEC_GOOD)
+    full.update(kw)
+    assert binding.mk_attn_decode_paged(**full) == want

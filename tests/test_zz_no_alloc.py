@@ -1,14 +1,21 @@
-"""The allocation-free decode entry point against the workspace one, on the GPU.
+"""The allocation-free decode entry point, on the GPU.
 
 mk_attn_decode_paged_noalloc serves callers that cannot allocate device
 memory (code running under an allocator that another runtime owns, inside
 host callbacks, or in plugins that must not grow the device heap): its split
 partials go to a fixed 16 MiB array that the library declares in device
 memory instead of a caller workspace.  These tests call it through the C ABI
-and check it against mk_attn_decode_paged with a workspace, within the decode
-tests' tolerances, on two calls in a row (the second sees what the first left
-in the shared array), and check that sizes needing more scratch than the
-array holds are refused before anything is launched.
+and check it
+  - against mk_attn_decode_paged with a workspace: both run the same kernels
+    with the same split plan, so the outputs must agree bit for bit (which
+    also holds them within the decode tests' tolerances);
+  - against the fp64 oracle, within the decode tests' tolerances;
+on two calls in a row: the second call has the same sizes but shorter
+sequences, so a merge that read partials the first call left in the shared
+array would show;
+  - that a warm call changes the device's free memory by nothing;
+  - that sizes needing more scratch than the array holds are refused before
+    anything is launched.
 
 The file name makes pytest collect it last."""
 import math
@@ -17,6 +24,7 @@ import numpy as np
 import pytest
 import torch
 
+import oracle
 from paper_2609_04523_gb300 import binding
 from paper_2609_04523_gb300 import workloads as W
 
@@ -64,8 +72,10 @@ def _call_workspace(args, inp, o, lse, stream):
 
 
 def _compare(o, lse, o_ref, lse_ref, what):
-    o, o_ref = o.float().cpu().numpy(), o_ref.float().cpu().numpy()
-    lse, lse_ref = lse.double().cpu().numpy(), lse_ref.double().cpu().numpy()
+    o = o.float().cpu().numpy()
+    o_ref = np.asarray(o_ref.float().cpu().numpy() if torch.is_tensor(o_ref) else o_ref)
+    lse = lse.double().cpu().numpy()
+    lse_ref = np.asarray(lse_ref.double().cpu().numpy() if torch.is_tensor(lse_ref) else lse_ref)
     assert np.all(np.isfinite(o)), f"{what}: o has unwritten entries"
     fin = np.isfinite(lse_ref)
     assert np.array_equal(fin, np.isfinite(lse)), f"{what}: empty rows differ"
@@ -78,28 +88,59 @@ def _compare(o, lse, o_ref, lse_ref, what):
     assert lerr <= LSE_MAX_ABS, f"{what}: lse err {lerr:.3e}"
 
 
-def test_noalloc_matches_workspace_entry_on_two_calls_in_a_row():
-    """Two different decode steps, both with several KV splits, so both go
-    through the static scratch; the second is checked after the first has
-    left its partials there."""
-    cases = [
-        W.make_paged([5000, 1, 0, 2100], 16, 4, 128, 64, seed=901),
-        W.make_paged([3, 4000, 777], 24, 3, 64, 32, seed=902),
-    ]
+def _shorter(inp, lens):
+    """The same decode step with shorter sequences (same sizes and pages)."""
+    sl = torch.tensor(lens, dtype=torch.int32)
+    assert torch.all(sl <= inp.seq_lens)
+    return W.PagedInputs(inp.q, inp.k_cache, inp.v_cache, inp.page_table, sl, inp.scale)
+
+
+@pytest.mark.parametrize("case", [0, 1])
+def test_noalloc_matches_workspace_entry_and_oracle_on_two_calls_in_a_row(case):
+    """Two decode steps of the same sizes, both with several KV splits, so
+    both go through the static scratch; the second has shorter sequences and
+    is checked after the first has left its partials there."""
+    first = [W.make_paged([5000, 1, 0, 2100], 16, 4, 128, 64, seed=901),
+             W.make_paged([3, 4000, 777], 24, 3, 64, 32, seed=902)][case]
+    second = _shorter(first, [[300, 1, 0, 1000], [3, 129, 40]][case])
     stream = torch.cuda.current_stream().cuda_stream
-    for n, inp in enumerate(cases):
+    for n, inp in enumerate((first, second)):
         B, Hq, Hkv, D, ps, mp, _ = _sizes(inp)
         need = binding.mk_attn_decode_workspace_bytes(B, Hq, Hkv, D, ps, mp)
-        assert 0 < need <= binding.DECODE_STATIC_SCRATCH_BYTES, f"case {n}: need {need}"
+        assert 0 < need <= binding.DECODE_STATIC_SCRATCH_BYTES, f"call {n + 1}: need {need}"
         args = _device_args(inp)
-        o_ref, lse_ref = _outputs(args[0])
-        st, _ws = _call_workspace(args, inp, o_ref, lse_ref, stream)
+        o_ws, lse_ws = _outputs(args[0])
+        st, _ws = _call_workspace(args, inp, o_ws, lse_ws, stream)
         assert st == binding.MK_OK, binding.mk_attn_error_string(st)
         o, lse = _outputs(args[0])
         st = _call_noalloc(args, inp, o, lse, stream)
         assert st == binding.MK_OK, binding.mk_attn_error_string(st)
         assert binding.mk_attn_check_status(stream) == binding.MK_OK
-        _compare(o, lse, o_ref, lse_ref, f"call {n + 1}")
+        what = f"case {case} call {n + 1}"
+        assert torch.equal(o.view(torch.int16), o_ws.view(torch.int16)), f"{what}: o differs"
+        assert torch.equal(lse, lse_ws), f"{what}: lse differs"
+        _compare(o, lse, o_ws, lse_ws, what + " vs workspace entry")
+        o_ref, lse_ref = oracle.decode_paged(inp.q, inp.k_cache, inp.v_cache, inp.page_table,
+                                             inp.seq_lens, inp.scale)
+        _compare(o, lse, o_ref, lse_ref, what + " vs oracle")
+
+
+def test_warm_noalloc_call_allocates_nothing():
+    """After a first call (which looks up the scratch address and loads the
+    library's decode kernels), a call changes the device's free memory by
+    nothing."""
+    inp = W.make_paged([3000, 17, 900], 16, 4, 128, 64, seed=904)
+    args = _device_args(inp)
+    o, lse = _outputs(args[0])
+    stream = torch.cuda.current_stream().cuda_stream
+    assert _call_noalloc(args, inp, o, lse, stream) == binding.MK_OK
+    torch.cuda.synchronize()
+    free0, _ = torch.cuda.mem_get_info()
+    assert _call_noalloc(args, inp, o, lse, stream) == binding.MK_OK
+    torch.cuda.synchronize()
+    free1, _ = torch.cuda.mem_get_info()
+    assert free1 == free0, f"free device memory moved by {free0 - free1} bytes"
+    assert binding.mk_attn_check_status(stream) == binding.MK_OK
 
 
 def test_noalloc_refuses_sizes_beyond_its_scratch():
