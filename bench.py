@@ -31,6 +31,11 @@ dK/dV kernel, timed alone, against the bf16 tensor roofline.
 576-wide latent cache, values its first 512 components, page_size=64) in HBM
 GB/s of algorithmic bytes, with its matmul TFLOP/s beside it.
 
+--workload hostcopy measures what bounds the end-to-end figures: pinned host
+to device and device to host copy bandwidth (100 MiB copies, one stream per
+direction, each direction alone and both at once), in GB/s.  It runs no
+kernel of the library.
+
 --impl reference times the fp64 CPU oracle on bounded row samples of the same
 workload (the whole step for decode, one sequence for the backward pass,
 leading sequences for the latent decode step; rank 0 only; other ranks exit
@@ -77,7 +82,7 @@ def parse_args():
     ap.add_argument("--settle-s", type=float, default=2.5,
                     help="seconds of untimed back-to-back steps before the warm-up")
     ap.add_argument("--workload", default="prefill",
-                    choices=["prefill", "decode", "backward", "mla"],
+                    choices=["prefill", "decode", "backward", "mla", "hostcopy"],
                     help="prefill: the attention forward pass (--config); decode: one paged "
                          "decode step (the decode workload below)")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
@@ -1323,6 +1328,71 @@ def run_mla_reference(args, rank: int):
     }
 
 
+# ------------------------------------------------------- host link copies
+
+HOSTCOPY_METRIC = "pinned host-device copy GB/s (what bounds the end-to-end figures)"
+
+
+def run_hostcopy(args, rank: int, world: int, local_rank: int):
+    """Pinned host -> device and device -> host bandwidth with torch copies on
+    dedicated streams: each direction alone, then both at once.  A step is one
+    100 MiB copy per direction; CUDA events on the copy streams."""
+    import torch
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    n = 100 << 20
+    h_src = torch.empty(n, dtype=torch.uint8).pin_memory()
+    h_src.fill_(1)
+    h_dst = torch.empty(n, dtype=torch.uint8).pin_memory()
+    d_a = torch.empty(n, dtype=torch.uint8, device=dev)
+    d_b = torch.empty(n, dtype=torch.uint8, device=dev)
+    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+
+    def timed(run_in: bool, run_out: bool) -> float:
+        for _ in range(args.warmup):
+            if run_in:
+                with torch.cuda.stream(s_in):
+                    d_a.copy_(h_src, non_blocking=True)
+            if run_out:
+                with torch.cuda.stream(s_out):
+                    h_dst.copy_(d_b, non_blocking=True)
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(torch.cuda.current_stream(dev))
+        s_in.wait_stream(torch.cuda.current_stream(dev))
+        s_out.wait_stream(torch.cuda.current_stream(dev))
+        for _ in range(args.steps):
+            if run_in:
+                with torch.cuda.stream(s_in):
+                    d_a.copy_(h_src, non_blocking=True)
+            if run_out:
+                with torch.cuda.stream(s_out):
+                    h_dst.copy_(d_b, non_blocking=True)
+        torch.cuda.current_stream(dev).wait_stream(s_in)
+        torch.cuda.current_stream(dev).wait_stream(s_out)
+        e1.record(torch.cuda.current_stream(dev))
+        torch.cuda.synchronize(dev)
+        return e0.elapsed_time(e1) / args.steps  # ms per step
+
+    ms_in = timed(True, False)
+    ms_out = timed(False, True)
+    ms_both = timed(True, True)
+    if rank != 0:
+        return None
+    gbs = lambda ms: round(n / (ms * 1e-3) / 1e9, 1)
+    return {
+        "metric": HOSTCOPY_METRIC, "value": gbs(ms_in), "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_in, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
+        "data": "synthetic (100 MiB pinned host buffer)",
+        "config": {"workload": "pinned copies of 100 MiB, torch copy_ on dedicated streams",
+                   "h2d_gbs": gbs(ms_in), "d2h_gbs": gbs(ms_out),
+                   "both_at_once_each_gbs": gbs(ms_both),
+                   "note": "value = host to device alone; no kernel of this library runs"},
+        "gpu_launches": 0,
+    }
+
+
 # ----------------------------------------------------------- reference arm
 
 def run_reference(args, rank: int):
@@ -1370,6 +1440,15 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.workload == "hostcopy":
+        if args.impl == "reference":
+            print(json.dumps({"impl": "reference", "unavailable": "hostcopy measures the host "
+                              "link only; there is no reference program for it"}), flush=True)
+            return
+        line = run_hostcopy(args, rank, world, int(os.environ.get("LOCAL_RANK", "0")))
+        if line is not None:
+            print(json.dumps(line), flush=True)
+        return
     if args.impl == "reference":
         if args.workload == "decode":
             line = run_decode_reference(args, rank)

@@ -58,7 +58,10 @@ typedef enum {
  *                  mk_attn_check_status reports (MK_OK, MK_ERR_TIMEOUT,
  *                  MK_ERR_INVALID_ARG, MK_ERR_BOUNDS, MK_ERR_CUDA) instead of
  *                  MK_OK: a device-side error is then tied to the call that
- *                  caused it.  Such calls are no longer asynchronous.
+ *                  caused it.  Such calls are no longer asynchronous, so the
+ *                  check mode cannot be used while a stream is being captured
+ *                  into a CUDA graph (the synchronisation would fail the call
+ *                  with MK_ERR_CUDA).
  *   MK_DEBUG       compile definition of the check build of this library
  *                  (libmk_attn_debug.so).  Every kernel then checks the index
  *                  of each global-memory store of its outputs, partials and
