@@ -36,7 +36,8 @@ def check_fwd(o, lse, o_ref, lse_ref):
     assert float(np.max(np.abs(lse - lse_ref))) <= 1e-3
 
 
-KNOBS = [dict(ctas=1), dict(ctas=37), dict(ctas=300), dict(schedule=binding.SCHED_ROUND_ROBIN),
+KNOBS = [dict(ctas=1), dict(ctas=37), dict(ctas=300), dict(schedule=binding.SCHED_SNAKE),
+         dict(schedule=binding.SCHED_ROUND_ROBIN),
          dict(schedule=binding.SCHED_BLOCKED), dict(ctas=64, schedule=binding.SCHED_BLOCKED),
          dict(schedule=binding.SCHED_DYNAMIC), dict(ctas=1, schedule=binding.SCHED_DYNAMIC),
          dict(ctas=37, schedule=binding.SCHED_DYNAMIC)]
@@ -158,7 +159,8 @@ def test_dynamic_schedule_counters_reset_over_many_launches_and_two_streams():
     dev = torch.device("cuda")
     q, k, v, _ = W.make_qkv(1, 4, 2, 2048, 64, seed=932)
     q, k, v = q.to(dev), k.to(dev), v.to(dev)
-    o_ref, lse_ref = binding.attn_fwd(q, k, v, causal=True, scale=0.125)
+    with binding.tuning(schedule=binding.SCHED_SNAKE):
+        o_ref, lse_ref = binding.attn_fwd(q, k, v, causal=True, scale=0.125)
     streams = [torch.cuda.Stream(), torch.cuda.Stream()]
     for st in streams:
         st.wait_stream(torch.cuda.current_stream())
