@@ -228,6 +228,21 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(self.samples), "source": self.source}
 
 
+# GPU cycles of torch's bounded spin kernel before each timed loop: about 5 ms.
+HEAD_START_CYCLES = 10_000_000
+HEAD_START_NOTE = "a 5 ms GPU spin (outside the events) before the first step keeps the host ahead"
+
+
+def head_start():
+    """Keeps the GPU busy for a few milliseconds, outside every event pair,
+    while the host enqueues the first timed steps: with the GPU idle at the
+    start of the loop, a host delay (the clock sampler starting, the Python
+    call path of a step) would otherwise show up inside the first steps'
+    events as GPU idle time."""
+    import torch
+    torch.cuda._sleep(HEAD_START_CYCLES)
+
+
 def clocks_rejected(c) -> bool:
     if c is None:
         return False
@@ -428,6 +443,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
             torch.distributed.barrier()
         torch.cuda.synchronize(dev)
         with ClockSampler(pci_bus_id, local_rank) as cs:
+            head_start()
             for i in range(args.steps):
                 flush.zero_()
                 starts[i].record(stream)
@@ -530,7 +546,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
             "flop_convention": "4*D*L^2 per sequence and head, halved when causal",
             "pct_of_nominal_2250_tflops": round(100.0 * per_launch_tflops / NOMINAL_BF16_TFLOPS, 2),
             "l2": "flushed before every timed step (256 MiB device write, outside the event pair)",
-            "timing": "CUDA events around each launch on the launching stream; sum over steps",
+            "timing": "CUDA events around each launch on the launching stream; sum over steps; " + HEAD_START_NOTE,
             "settle": f"{settle_steps} untimed back-to-back steps ({args.settle_s} s) before the "
                       f"{args.warmup} warm-up steps",
             "ms_per_step_x_sm_mhz": clock_normalised(ms_per_step, clocks),
@@ -653,6 +669,7 @@ def run_decode(args, rank: int, world: int, local_rank: int):
             torch.distributed.barrier()
         torch.cuda.synchronize(dev)
         with ClockSampler(pci_bus_id, local_rank) as cs:
+            head_start()
             for i in range(args.steps):
                 flush.zero_()
                 starts[i].record(stream)
@@ -744,7 +761,7 @@ def run_decode(args, rank: int, world: int, local_rank: int):
             "l2": "flushed before every timed step (256 MiB device write, outside the event pair); "
                   "the cache (%.2f GB) is far larger than L2" % (4 * sum(lens) * Hkv * D / 1e9),
             "timing": "CUDA events around each call (decode kernel and, with several KV splits, "
-                      "the merge kernel) on the launching stream; sum over steps",
+                      "the merge kernel) on the launching stream; sum over steps; " + HEAD_START_NOTE,
             "parallelism": f"replicas x{world} (independent workloads per GPU)",
         },
         "roofline": {
@@ -898,6 +915,7 @@ def run_backward(args, rank: int, world: int, local_rank: int):
             torch.distributed.barrier()
         torch.cuda.synchronize(dev)
         with ClockSampler(pci_bus_id, local_rank) as cs:
+            head_start()
             for i in range(args.steps):
                 flush.zero_()
                 starts[i].record(stream)
@@ -1009,7 +1027,7 @@ def run_backward(args, rank: int, world: int, local_rank: int):
                           "dkdv": round(t_dkdv * 1e3, 5), "dq": round(t_dq * 1e3, 5)},
             "l2": "flushed before every timed step (256 MiB device write, outside the event pair)",
             "timing": "CUDA events around each call (dQ kernel, which also computes Delta, then dK/dV) on the launching "
-                      "stream; sum over steps; each kernel also timed alone the same way",
+                      "stream; sum over steps; each kernel also timed alone the same way; " + HEAD_START_NOTE,
             "parallelism": f"replicas x{world} (independent workloads per GPU)",
         },
         "roofline": {
@@ -1164,6 +1182,7 @@ def run_mla(args, rank: int, world: int, local_rank: int):
             torch.distributed.barrier()
         torch.cuda.synchronize(dev)
         with ClockSampler(pci_bus_id, local_rank) as cs:
+            head_start()
             for i in range(args.steps):
                 flush.zero_()
                 starts[i].record(stream)
@@ -1261,7 +1280,7 @@ def run_mla(args, rank: int, world: int, local_rank: int):
             "l2": "flushed before every timed step (256 MiB device write, outside the event pair); "
                   "the cache (%.2f GB) is larger than L2" % (2 * sum(lens) * 576 / 1e9),
             "timing": "CUDA events around each call (latent decode kernel and, with several KV "
-                      "splits, the merge kernel) on the launching stream; sum over steps",
+                      "splits, the merge kernel) on the launching stream; sum over steps; " + HEAD_START_NOTE,
             "parallelism": f"replicas x{world} (independent workloads per GPU)",
         },
         "roofline": {
