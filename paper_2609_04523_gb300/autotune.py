@@ -45,22 +45,29 @@ def candidates(space: dict):
         yield dict(zip(names, values))
 
 
+# GPU cycles of torch's bounded spin kernel before the timed calls: about 5 ms.
+HEAD_START_CYCLES = 10_000_000
+
+
 def time_call(fn, steps: int, warmup: int, flush, stream) -> float:
-    """Mean CUDA-event time of fn() in ms, L2 flushed before each call."""
+    """Mean CUDA-event time of fn() in ms, L2 flushed before each call.  All
+    calls are enqueued behind a short GPU spin and synchronised once, so the
+    host stays ahead and no call's events include GPU idle time."""
     import torch
     for _ in range(warmup):
         flush.zero_()
         fn()
-    ms = []
-    for _ in range(steps):
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    torch.cuda.synchronize()
+    torch.cuda._sleep(HEAD_START_CYCLES)
+    for a, b in zip(starts, ends):
         flush.zero_()
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
         fn()
         b.record(stream)
-        b.synchronize()
-        ms.append(a.elapsed_time(b))
-    return statistics.mean(ms)
+    torch.cuda.synchronize()
+    return statistics.mean(a.elapsed_time(b) for a, b in zip(starts, ends))
 
 
 def make_step(workload: str, config: int, dev):
