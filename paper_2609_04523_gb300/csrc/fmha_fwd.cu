@@ -728,16 +728,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         // branch-free: a branch inside it would stop the scheduler from
         // overlapping the MUFU latencies of consecutive keys.
         auto load_scores = [&](float (&s)[kTile]) {
-          uint32_t raw[4][32];
-#pragma unroll
-          for (int c = 0; c < 4; ++c) tmem_ld_32x32b_x32(t_s + c * 32, raw[c]);
+          uint32_t raw[kTile];
+          tmem_ld_32x32b_x128(t_s, raw);
           tmem_ld_wait();
+          reg_fence_n(raw);
 #pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            reg_fence(raw[c]);
-#pragma unroll
-            for (int e = 0; e < 32; ++e) s[c * 32 + e] = __uint_as_float(raw[c][e]);
-          }
+          for (int c = 0; c < kTile; ++c) s[c] = __uint_as_float(raw[c]);
           if (neg_scale) {
 #pragma unroll
             for (int c = 0; c < kTile; ++c) s[c] = -s[c];
