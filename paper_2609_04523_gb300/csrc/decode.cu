@@ -442,6 +442,9 @@ __global__ void __launch_bounds__(kThreads, MH > 4 ? 2 : 3)
 // evaluated relative to the largest lse_s.  One warp per (b, h).
 template <int D>
 __global__ void __launch_bounds__(128) merge_kernel(const Params p) {
+  // Launched as a programmatic dependent of the decode kernel: nothing is read
+  // before that kernel's partials are complete and visible.
+  griddep_wait();
   constexpr int NDL = D / 32;
   const int row = blockIdx.x * 4 + threadIdx.x / 32;  // b * Hq + h
   if (row >= p.B * p.Hq) return;
@@ -557,8 +560,9 @@ static int launch(const CUtensorMap &tk, const CUtensorMap &tv, const Params &p,
   decode_kernel<D, MH><<<grid, kThreads, sm, st>>>(tk, tv, p);
   if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
   if (p.n_splits > 1) {
-    merge_kernel<D><<<(p.B * p.Hq + 3) / 4, 128, 0, st>>>(p);
-    if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
+    // Scheduled while the decode grid drains; it waits for the partials itself.
+    DependentLaunch dl(dim3((p.B * p.Hq + 3) / 4), dim3(128), 0, st);
+    if (cudaLaunchKernelEx(&dl.cfg, merge_kernel<D>, p) != cudaSuccess) return MK_ERR_CUDA;
   }
   return MK_OK;
 }

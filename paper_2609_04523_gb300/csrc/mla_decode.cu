@@ -462,6 +462,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 // o_s = (sum over its keys of exp(s_j) c_j) / exp(lse_s), stored with lse_s
 // at component 512 of a 516-float row.
 __global__ void __launch_bounds__(128) mla_merge_kernel(const Params p) {
+  // Launched as a programmatic dependent of the latent decode kernel: nothing
+  // is read before that kernel's partials are complete and visible.
+  griddep_wait();
   constexpr int NDL = kDv / 32;
   const int row = blockIdx.x * 4 + threadIdx.x / 32;  // b * Hq + h
   if (row >= p.B * p.Hq) return;
@@ -638,8 +641,9 @@ static int mla_decode_impl(const void *q, const void *cache, const int32_t *page
   mla::mla_decode_kernel<<<grid, mla::kThreads, mla::kSmemBytes, st>>>(tq, tc, p);
   if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
   if (p.n_splits > 1) {
-    mla::mla_merge_kernel<<<(B * Hq + 3) / 4, 128, 0, st>>>(p);
-    if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
+    // Scheduled while the decode grid drains; it waits for the partials itself.
+    DependentLaunch dl(dim3((B * Hq + 3) / 4), dim3(128), 0, st);
+    if (cudaLaunchKernelEx(&dl.cfg, mla::mla_merge_kernel, p) != cudaSuccess) return MK_ERR_CUDA;
   }
   return MK_OK;
 }

@@ -115,6 +115,15 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volati
   }
 }
 
+// Programmatic dependent launch: a kernel launched with programmatic stream
+// serialization may be scheduled before the kernel ahead of it on the stream
+// has finished; griddep_wait() blocks until that kernel has completed and its
+// memory operations are visible.  In a kernel launched without it, it returns
+// at once.
+__device__ __forceinline__ void griddep_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
 // Warp-wide wait, called by all 32 lanes of a converged warp: one poll and
 // one vote on the fast path (the phase has already completed), the bounded
 // spin otherwise.  Returns the same value in every lane.

@@ -42,6 +42,29 @@ inline bool encode_tokens_heads_dim(CUtensorMap *map, const void *base, uint64_t
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Launch configuration of a kernel that follows another kernel of the same
+// call on `stream` and reads its results: with programmatic stream
+// serialization it may be scheduled while the first kernel drains, and it calls
+// griddep_wait() before reading anything.  Use as a local: cfg.attrs points
+// into the object.
+struct DependentLaunch {
+  cudaLaunchConfig_t cfg;
+  cudaLaunchAttribute attr[1];
+  DependentLaunch(dim3 grid, dim3 block, size_t smem, cudaStream_t stream) {
+    cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+  }
+  DependentLaunch(const DependentLaunch &) = delete;
+  DependentLaunch &operator=(const DependentLaunch &) = delete;
+};
+
 // The process-wide launch tuning (mk_attn_set_tuning), defaults applied.
 mk_attn_tuning current_tuning();
 
