@@ -72,6 +72,21 @@ typedef enum {
  */
 
 /*
+ * Streams and CUDA graphs.  Every entry point only enqueues work on the
+ * caller's stream (host-side checks and tensor-map encoding aside), so a call
+ * can be captured into a CUDA graph and replayed, with these conditions:
+ *   - make one call of each entry point and head dimension outside the
+ *     capture first (it sets the kernels' shared-memory limits once per
+ *     device);
+ *   - no check mode (MK_ATTN_DEBUG) during the capture;
+ *   - mk_attn_decode_paged_noalloc: see its scratch lookup below;
+ *   - MK_SCHED_DYNAMIC (mk_attn_tuning): see the schedule's counter slot.
+ * Where one call launches two kernels (the decode and latent decode merges),
+ * the second is a programmatic dependent launch: it may be scheduled while the
+ * first drains and waits on the device for its results.
+ */
+
+/*
  * mk_attn_fwd -- attention forward pass (causal or not, GQA, optional varlen).
  *
  * Arguments (all pointers are DEVICE pointers owned by the caller):
