@@ -89,13 +89,19 @@ struct KernelCfg {
   static constexpr int kStages = (D == 128) ? 2 : 4;
   static constexpr int kHalves = D / kBoxCols;      // swizzle boxes per tile
   static constexpr int kTileBytes = kTile * D * 2;  // one Q, K or V tile
+  // D = 64: o is staged per warp (32 rows x 64 columns, 4 KB, 128-byte
+  // swizzle) and written by TMA stores; 32 KB for the eight softmax warps.
+  // At D = 128 there is no room for it, and the rows are stored directly.
+  static constexpr bool kStageO = (D == 64);
   static constexpr int kOffQ = 0;                   // Q_A, then Q_B
   static constexpr int kOffK = 2 * kTileBytes;
   static constexpr int kOffV = kOffK + kStages * kTileBytes;
-  static constexpr int kOffCu = kOffV + kStages * kTileBytes;
+  static constexpr int kOffStage = kOffV + kStages * kTileBytes;
+  static constexpr int kOffCu = kOffStage + (kStageO ? 8 * 4096 : 0);
   static constexpr int kOffLvl = kOffCu + kCuCache * 4;  // (kMaxLevels + 2) ints
   static constexpr int kOffCtl = kOffLvl + ((kMaxLevels + 2) * 4 + 15) / 16 * 16;
   static constexpr int kSmemBytes = kOffCtl + 512 + 1024;  // + control block + alignment slack
+  static_assert(kSmemBytes <= 232448, "shared memory per block");
 };
 
 struct Unit {
@@ -333,7 +339,8 @@ template <int D, bool VL>
 __global__ void __launch_bounds__(kThreads, 1)
     mk_attn_fwd_persistent(const __grid_constant__ CUtensorMap tm_q,
                     const __grid_constant__ CUtensorMap tm_k,
-                    const __grid_constant__ CUtensorMap tm_v, const Params p) {
+                    const __grid_constant__ CUtensorMap tm_v,
+                    const __grid_constant__ CUtensorMap tm_o, const Params p) {
   using C = KernelCfg<D>;
   constexpr int NS = C::kStages;
 
@@ -827,9 +834,51 @@ __global__ void __launch_bounds__(kThreads, 1)
           row_valid &&
           dbg_in_range(tok, VL ? (int64_t)p.S : (int64_t)p.B * p.S, &g_status) &&
           dbg_in_range(w.hq, p.Hq, &g_status);
+      // D = 64, a tile that lies inside its sequence: each warp stages its 32
+      // rows in the 128-byte swizzle and stores them with one TMA store, which
+      // writes whole lines and keeps the stores off the load/store pipe.  A
+      // tile cut by the end of its sequence keeps the per-row stores.
+      const int64_t tok0 = (int64_t)w.seq_start + qt * kTile;
+      const bool tile_store =
+          C::kStageO && qt * kTile + kTile <= w.len &&
+          dbg_in_range(tok0 + kTile - 1, VL ? (int64_t)p.S : (int64_t)p.B * p.S, &g_status) &&
+          dbg_in_range(w.hq, p.Hq, &g_status);
+      if (tile_store) {
+        const int wq = warp % 4;
+        uint8_t *wbox = smem + C::kOffStage + (X * 4 + wq) * 4096;
+        const uint32_t row_a = smem_addr(wbox) + lane_id() * 128;
+        uint32_t o_raw[2][32];
+        tmem_ld_32x32b_x32(t_o, o_raw[0]);
+        tmem_ld_32x32b_x32(t_o + 32, o_raw[1]);
+        // The box is free once this warp's previous store has read it.
+        if (lane_id() == 0) bulk_wait_group_read_all();
+        __syncwarp();
+        tmem_ld_wait();
+#pragma unroll
+        for (int cc = 0; cc < 2; ++cc) {
+          reg_fence(o_raw[cc]);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            // 16-byte chunk j = 4 cc + e of this row goes to position j ^ (row % 8).
+            const uint32_t a = row_a + ((((cc * 4 + e) ^ (lane_id() & 7)) & 7) << 4);
+            const float *f = reinterpret_cast<const float *>(&o_raw[cc][8 * e]);
+            st_shared_v4(a, pack_bf16x2(f[0] * inv_l, f[1] * inv_l),
+                         pack_bf16x2(f[2] * inv_l, f[3] * inv_l),
+                         pack_bf16x2(f[4] * inv_l, f[5] * inv_l),
+                         pack_bf16x2(f[6] * inv_l, f[7] * inv_l));
+          }
+        }
+        fence_proxy_async_shared();
+        __syncwarp();
+        if (lane_id() == 0) {
+          tma_store_3d(&tm_o, wbox, 0, w.hq, (int32_t)tok0 + wq * 32, pol_o);
+          bulk_commit_group();
+        }
+        __syncwarp();
+      }
       uint4 *dst = reinterpret_cast<uint4 *>(p.o + (tok * p.Hq + w.hq) * (int64_t)D);
 #pragma unroll
-      for (int c = 0; c < D / 32; ++c) {
+      for (int c = 0; c < (tile_store ? 0 : D / 32); ++c) {
         uint32_t o_raw[32];
         tmem_ld_32x32b_x32(t_o + c * 32, o_raw);
         tmem_ld_wait();
@@ -865,6 +914,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     if (!ok) *abort = 1;
+    // Every TMA store of o this warp issued completes before the CTA releases
+    // its shared memory.
+    if (C::kStageO && lane_id() == 0) bulk_wait_group_all();
   }
 
   tc_fence_before_sync();
@@ -908,8 +960,9 @@ template <int D, bool VL>
 static int launch(const void *q, const void *k, const void *v, const Params &p, int64_t tokens,
                   cudaStream_t stream) {
   using C = KernelCfg<D>;
-  CUtensorMap tq, tk, tv;
+  CUtensorMap tq, tk, tv, to;
   if (!encode_tokens_heads_dim(&tq, q, tokens, p.Hq, D, kTile) ||
+      !encode_tokens_heads_dim(&to, p.o, tokens, p.Hq, D, 32) ||
       !encode_tokens_heads_dim(&tk, k, tokens, p.Hkv, D, kTile) ||
       !encode_tokens_heads_dim(&tv, v, tokens, p.Hkv, D, kTile))
     return MK_ERR_CUDA;
@@ -934,7 +987,7 @@ static int launch(const void *q, const void *k, const void *v, const Params &p, 
   const int ctas = tune.ctas > 0 ? tune.ctas : di.sm_count;
   const int grid = p.n_units < ctas ? p.n_units : ctas;
   mark_launched(kFamFwd);
-  mk_attn_fwd_persistent<D, VL><<<grid, kThreads, C::kSmemBytes, stream>>>(tq, tk, tv, p);
+  mk_attn_fwd_persistent<D, VL><<<grid, kThreads, C::kSmemBytes, stream>>>(tq, tk, tv, to, p);
   return cudaGetLastError() == cudaSuccess ? MK_OK : MK_ERR_CUDA;
 }
 
