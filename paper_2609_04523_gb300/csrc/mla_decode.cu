@@ -10,27 +10,41 @@
 //   lse[b,h]    = ln sum_j exp(scale * q[b,h,:] . c_j)
 // with position j in slot j % page_size of page page_table[b, j / page_size].
 //
-// All heads share every key, so the step is a pair of dense contractions per
-// block of 128 keys and runs on tcgen05 with the query heads as the MMA's M
-// dimension (up to 128 heads per CTA, missing heads zero-filled by TMA):
-//   S  = Q C^T        M = heads, N = 128 keys, K = 576 (nine 64-wide chunks)
-//   O += P C[:, :dv]  M = heads, N = 64 value components per MMA, K = 128 keys
-// Capacity sets the shape.  Q (128 x 576 bf16 = 144 KB) stays in shared
-// memory; the cache streams through a ring of five 16 KB chunk slots (128
-// keys x 64 components each), in the order the MMAs consume them: the nine
-// key chunks of block n+1, then the value chunks of block n (the same rows,
-// read again from L2).  O for 128 heads x 512 components would fill TMEM's
-// 512 columns, so the value dimension is split over two CTAs (each computes
-// S itself and keeps a 256-column O); TMEM is S double-buffered (2 x 128
-// columns) + O (256 columns).  Softmax: base 2, one thread per head row, the
-// lazy rescale of the forward kernel (O in TMEM is rescaled only when the
-// row max rises by more than 8); P (bf16) overwrites the first 64 columns of
-// its S buffer and is the TMEM A operand of the P.V MMAs.  KV splits with a
+// All heads share every key, so a block of 64 keys is a pair of dense
+// contractions on tcgen05 with the query heads as the MMA's M dimension (up to
+// 128 heads, missing heads zero):
+//   S  = Q C^T        M = heads, N = 64 keys, K = 576 (nine 64-wide chunks)
+//   O += P C[:, :dv]  M = heads, N = 64 value components per MMA, K = 64 keys
+// O for 128 heads x 512 components fills TMEM's 512 columns, so two CTAs
+// share the work, as a cluster of two: CTA h keeps the value half
+// 256 h .. 256 h + 255 of O, loads only the cache chunks it needs for that half
+// (chunks 4 h .. 4 h + 3, and CTA 0 also the rotary chunk 8), and computes the
+// part of S over those chunks.  The two CTAs exchange their partial scores
+// (128 x 64 fp32 per block) through distributed shared memory -- each thread
+// sends its row with asynchronous stores that complete on an mbarrier of the
+// partner -- and both add them (the sum is the same in both CTAs), so each
+// cached byte crosses from L2 into one SM only, and each CTA's value chunks
+// are the key chunks it already holds.  S over the four TMEM
+// chunks reads Q from TMEM (the TS form, at the tensor rate for N = 64); CTA
+// 0's rotary chunk reads Q from shared memory.
+//
+// TMEM (512 columns): partial S, then P (bf16, first 32 columns), double
+// buffered at 0 and 64; the CTA's four Q chunks at 128 (32 columns each);
+// O (256 columns) at 256.  Shared memory: CTA 0's Q chunk 8 (16 KB), a ring
+// of three block slots (up to five 8 KB chunks each), two 32 KB exchange
+// slots written by the partner CTA.
+//
+// Softmax: base 2, one thread per head row, lazy rescale (O in TMEM is
+// rescaled only when the row max rises by more than 8).  KV splits with a
 // log-sum-exp merge fill the GPU at small batch, as in the paged decode step.
 //
-// Roles: warps 0-3 softmax and epilogue (thread = head row = TMEM lane),
-// warp 4 tcgen05 MMA issuer, warp 5 TMA producer.  One CTA per SM (shared
-// memory), persistent only within its split.
+// Roles: warps 0-3 softmax, exchange and epilogue (thread = head row = TMEM
+// lane), warp 4 tcgen05 MMA issuer, warp 5 TMA producer.  One CTA per SM.
+// Every wait is bounded; a CTA that gives up records a timeout, and its
+// partner's waits for it run out in turn, so both reach the final cluster
+// barrier.  A CTA's last asynchronous store to its partner is either waited
+// for by the partner or followed by a wait of its own that runs out (2 s)
+// before it reaches that barrier, so no store lands after the partner left.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
@@ -49,31 +63,38 @@ namespace mla {
 constexpr int kDqk = MK_MLA_DQK;          // 576
 constexpr int kDv = MK_MLA_DV;            // 512
 constexpr int kChunk = 64;                // components per chunk (one 128-byte swizzle row)
-constexpr int kChunksK = kDqk / kChunk;   // 9
 constexpr int kDvCta = kDv / 2;           // 256 value components per CTA
 constexpr int kChunksV = kDvCta / kChunk; // 4
 constexpr int kHeads = 128;               // M: heads per CTA
-constexpr int kBlock = 128;               // keys per block (N of S)
-constexpr int kChunkBytes = kBlock * kChunk * 2;  // 16 KB: 128 rows x 128 B
-constexpr int kQBytes = kChunksK * kHeads * kChunk * 2;  // 144 KB
-constexpr int kSlots = 5;
-constexpr int kOffRing = kQBytes;
-constexpr int kOffCtl = kOffRing + kSlots * kChunkBytes;
+constexpr int kBlock = 64;                // keys per block (N of S)
+constexpr int kChunkBytes = kBlock * kChunk * 2;   // 8 KB: 64 rows x 128 B
+constexpr int kQChunkBytes = kHeads * kChunk * 2;  // 16 KB
+constexpr int kMaxChunksCta = 5;          // CTA 0: chunks 0-3 and 8; CTA 1: chunks 4-7
+constexpr int kSlotBytes = kMaxChunksCta * kChunkBytes;
+constexpr int kSlots = 3;
+constexpr int kExchBytes = kHeads * kBlock * 4;    // 32 KB: one block's partial scores
+constexpr int kOffQ8 = 0;
+constexpr int kOffRing = kQChunkBytes;
+constexpr int kOffExch = kOffRing + kSlots * kSlotBytes;
+constexpr int kOffCtl = kOffExch + 2 * kExchBytes;
 constexpr int kSmemBytes = kOffCtl + 256 + 1024;
 static_assert(kSmemBytes <= 232448, "shared memory per CTA");
 constexpr int kThreads = 192;
 constexpr int kMmaWarp = 4, kLoadWarp = 5;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColS = 0;      // S buffer X at kColS + 128 X
+constexpr uint32_t kColS = 0;      // S buffer x at kColS + 64 x
+constexpr uint32_t kColQ = 128;    // TMEM Q chunk j at kColQ + 32 j (bf16 pairs)
 constexpr uint32_t kColO = 256;    // O: 256 columns
 constexpr float kRescaleThreshold = 8.0f;
 
 __device__ int g_status = 0;
 
 struct Ctl {
-  uint64_t q_full;
+  uint64_t q_full, qt_full;
   uint64_t slot_full[kSlots], slot_empty[kSlots];
   uint64_t s_full[2], p_full[2], pv_done[2];
+  uint64_t exch_full[2];   // the partner's partial scores of block n are here (32 KB tx)
+  uint64_t exch_empty[2];  // the partner has read this CTA's partial scores
   uint64_t mma_drained;
   uint32_t tmem_base;
   int abort;
@@ -81,6 +102,7 @@ struct Ctl {
 static_assert(sizeof(Ctl) <= 256, "control block");
 
 struct Params {
+  const uint16_t *q;          // bf16 [B, Hq, 576]
   const int32_t *page_table;  // [B, max_pages]
   const int32_t *seq_lens;    // [B]
   uint16_t *o;                // bf16 [B, Hq, 512]
@@ -109,12 +131,88 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, u
       : "memory");
 }
 
+// ---------------------------------------------------------- cluster helpers
+
+// The shared::cluster address of the partner CTA's copy of a local shared
+// memory address.
+__device__ __forceinline__ uint32_t peer_addr(uint32_t local, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
+  return r;
+}
+
+// All threads of both CTAs of the cluster (release / acquire).
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                   : "memory");
+}
+
+// Asynchronous store of 16 bytes into the partner CTA's shared memory,
+// counted (complete_tx) on the partner's mbarrier `remote_bar`.
+__device__ __forceinline__ void st_async_peer_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
+                                                 uint32_t d, uint32_t remote_bar) {
+  asm volatile(
+      "st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.b32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(
+          addr),
+      "r"(a), "r"(b), "r"(c), "r"(d), "r"(remote_bar)
+      : "memory");
+}
+
+__device__ __forceinline__ void ld_shared_v4(uint32_t addr, uint32_t &a, uint32_t &b, uint32_t &c,
+                                             uint32_t &d) {
+  asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(a), "=r"(b), "=r"(c), "=r"(d)
+               : "r"(addr)
+               : "memory");
+}
+
+// Relaxed arrival on an mbarrier of the partner CTA.  It follows local reads
+// whose values have already been consumed, so nothing remains to order; a
+// release arrival here costs about 1,000 clk per block (it waits for this
+// thread's outstanding remote stores).
+__device__ __forceinline__ void mbar_arrive_peer_relaxed(uint32_t remote_bar) {
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote_bar)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(done)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+
+// Bounded wait (as mbar_wait) with acquire at cluster scope: the phase was
+// completed by arrivals of the partner CTA, whose writes it publishes.
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t *bar, uint32_t parity,
+                                                  volatile int *abort) {
+  const uint32_t a = smem_addr(bar);
+  if (mbar_try_wait_cluster(a, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try_wait_cluster(a, parity)) return true;
+    if ((it & 255u) == 0) {
+      if (*abort) return false;
+      if (global_timer_ns() - t0 > kWaitLimitNs) {
+        *abort = 1;
+        return false;
+      }
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
     mla_decode_kernel(const __grid_constant__ CUtensorMap tm_q,
                       const __grid_constant__ CUtensorMap tm_c, const Params p) {
-  // blockIdx.x = 2 (b * head_groups + hg) + half, blockIdx.y = split: every
-  // sequence's first (largest) split is dispatched before any second one.
+  // blockIdx.x = 2 (b * head_groups + hg) + half: the two CTAs of a cluster
+  // (cluster rank = half) share (b, hg, split).  blockIdx.y = split.
   const int split = blockIdx.y, half = blockIdx.x & 1;
+  const uint32_t peer = (uint32_t)(half ^ 1);
   const int b = (blockIdx.x >> 1) / p.head_groups, hg = (blockIdx.x >> 1) % p.head_groups;
   const int PS = p.page_size;
   int L = p.seq_lens[b];
@@ -127,7 +225,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int nb = max(0, min(first + p.blocks_per_split, nblk_seq) - first);
   // Splits past the end of the sequence do nothing (the merge skips them);
   // split 0 always runs, so an empty sequence still gets o = 0, lse = -inf.
+  // Both CTAs of a cluster take the same branch.
   if (split > 0 && nb == 0) return;
+  // Chunks this CTA holds per block, in slot order: CTA 0 chunks 0-3 and the
+  // rotary chunk 8, CTA 1 chunks 4-7.  Positions 0-3 are the CTA's value
+  // chunks, whose Q chunks live in TMEM.
+  const int n_chunks = half == 0 ? 5 : 4;
+  auto chunk_of = [&](int j) { return half == 0 ? (j < 4 ? j : 8) : 4 + j; };
 
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_addr = smem_addr(smem_raw);
@@ -137,6 +241,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(&ctl->q_full, 1);
+    mbar_init(&ctl->qt_full, kHeads);
     for (int s = 0; s < kSlots; ++s) {
       mbar_init(&ctl->slot_full[s], 1);
       mbar_init(&ctl->slot_empty[s], 1);
@@ -145,6 +250,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&ctl->s_full[x], 1);
       mbar_init(&ctl->p_full[x], kHeads);
       mbar_init(&ctl->pv_done[x], 1);
+      mbar_init(&ctl->exch_full[x], 1);
+      mbar_init(&ctl->exch_empty[x], kHeads);
     }
     mbar_init(&ctl->mma_drained, 1);
     ctl->abort = 0;
@@ -157,40 +264,42 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before_sync();
   __syncthreads();
   tc_fence_after_sync();
+  // The partner's barriers are initialised before any arrival on them.
+  cluster_sync();
   const uint32_t tmem = ctl->tmem_base;
   volatile int *abort = &ctl->abort;
-  // Chunks a CTA consumes, in order: the nine key chunks of block n, then
-  // the four value chunks of block n - 1 (the MMAs' order), 13 per block.
-  const int n_steps = nb * (kChunksK + kChunksV);
 
   if (warp == kLoadWarp) {
     // ------------------------------------------------------------ producer
     bool ok = true;
     if (nb > 0) {
       if (elect_one()) {
-        tma_prefetch_desc(&tm_q);
         tma_prefetch_desc(&tm_c);
-        mbar_arrive_expect_tx(&ctl->q_full, kQBytes);
-        const uint64_t pol_q = l2_policy_evict_last();  // both value halves read it
-#pragma unroll 1
-        for (int c = 0; c < kChunksK; ++c)
-          tma_load_3d(smem + c * kHeads * kChunk * 2, &tm_q, &ctl->q_full, c * kChunk,
-                      hg * kHeads, b, pol_q);
+        if (half == 0) {
+          tma_prefetch_desc(&tm_q);
+          mbar_arrive_expect_tx(&ctl->q_full, kQChunkBytes);
+          tma_load_3d(smem + kOffQ8, &tm_q, &ctl->q_full, 8 * kChunk, hg * kHeads, b,
+                      l2_policy_evict_last());
+        }
       }
       __syncwarp();
     }
-    const uint64_t pol_c = l2_policy_evict_last();  // read again for the values
-    const int pages_per_block = kBlock / PS;  // 1..8
+    // Each cached chunk is read by one CTA, once.
+    const uint64_t pol_c = l2_policy_evict_first();
+    // A block is 64 / PS pages (PS <= 64) or half a page (PS = 128): one TMA
+    // load of min(PS, 64) rows per page piece and chunk.
+    const int rows_per_load = PS < kBlock ? PS : kBlock;
+    const int loads_per_block = kBlock / rows_per_load;  // 1..4
     const int n_pages_seq = (L + PS - 1) / PS;
     const int lane = lane_id();
-    // Physical page of page `lane` of block n (lanes < pages_per_block), one
+    // Physical page of piece `lane` of block n (lanes < loads_per_block), one
     // global load per lane per block, loaded one block ahead.  Pages past the
     // sequence end take the block's first page instead (finite rows, masked
-    // out), so every chunk moves the same number of bytes.
+    // out), so every slot moves the same number of bytes.
     auto block_pages = [&](int n) {
       int page = 0;
-      if (n < nb && lane < pages_per_block) {
-        const int page0 = (first + n) * pages_per_block;
+      if (n < nb && lane < loads_per_block) {
+        const int page0 = (int)((int64_t)(first + n) * kBlock / PS);
         const int lp = page0 + lane < n_pages_seq ? page0 + lane : page0;
         page = p.page_table[(int64_t)b * p.max_pages + lp];
         if (page < 0 || page >= p.num_pages) {
@@ -200,113 +309,102 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       return page;
     };
-    int t = 0;  // chunk step: the same order the MMA warp consumes
-    // One chunk (128 keys x 64 components at component offset 64 * chunk) of
-    // the block whose pages are in `pages` (lane i: page i).
-    auto load_chunk = [&](int pages, int chunk) {
-      const int s = t % kSlots;
-      ok = mbar_wait_all(&ctl->slot_empty[s], ((t / kSlots) & 1) ^ 1, abort);
-      if (!ok) return;
+    int pages_cur = block_pages(0);
+    for (int n = 0; ok && n < nb; ++n) {
+      const int pages_next = block_pages(n + 1);
+      const int s = n % kSlots;
+      ok = mbar_wait_all(&ctl->slot_empty[s], ((n / kSlots) & 1) ^ 1, abort);
+      if (!ok) break;
       int pg[kBlock / 16];
 #pragma unroll
-      for (int i = 0; i < kBlock / 16; ++i) pg[i] = __shfl_sync(0xffffffffu, pages, i);
+      for (int i = 0; i < kBlock / 16; ++i) pg[i] = __shfl_sync(0xffffffffu, pages_cur, i);
+      const int row0 = PS > kBlock ? (int)(((int64_t)(first + n) * kBlock) % PS) : 0;
       if (elect_one()) {
-        mbar_arrive_expect_tx(&ctl->slot_full[s], kChunkBytes);
-        uint8_t *dst = smem + kOffRing + s * kChunkBytes;
+        mbar_arrive_expect_tx(&ctl->slot_full[s], n_chunks * kChunkBytes);
+        uint8_t *dst = smem + kOffRing + s * kSlotBytes;
+        for (int j = 0; j < n_chunks; ++j)
 #pragma unroll
-        for (int i = 0; i < kBlock / 16; ++i)
-          if (i < pages_per_block)
-            tma_load_2d(dst + i * PS * 128, &tm_c, &ctl->slot_full[s], chunk * kChunk, pg[i] * PS,
-                        pol_c);
+          for (int i = 0; i < kBlock / 16; ++i)
+            if (i < loads_per_block)
+              tma_load_2d(dst + j * kChunkBytes + i * rows_per_load * 128, &tm_c,
+                          &ctl->slot_full[s], chunk_of(j) * kChunk, pg[i] * PS + row0, pol_c);
       }
       __syncwarp();
-      ++t;
-    };
-    int pages_prev = 0, pages_cur = block_pages(0);
-    for (int n = 0; ok && n <= nb; ++n) {
-      const int pages_next = block_pages(n + 1);
-      // The nine key chunks of block n, then the value chunks of block n-1.
-      if (n < nb)
-        for (int c = 0; ok && c < kChunksK; ++c) load_chunk(pages_cur, c);
-      if (n >= 1)
-        for (int c = 0; ok && c < kChunksV; ++c) load_chunk(pages_prev, half * kChunksV + c);
-      pages_prev = pages_cur;
       pages_cur = pages_next;
     }
     // Teardown: the loads issued land before the CTA exits.
-    if (nb > 0) drain_wait(&ctl->q_full, 0);
-    for (int t = max(0, n_steps - kSlots); t < n_steps; ++t)
-      drain_wait(&ctl->slot_full[t % kSlots], (t / kSlots) & 1);
+    if (nb > 0 && half == 0) drain_wait(&ctl->q_full, 0);
+    for (int n = max(0, nb - kSlots); n < nb; ++n)
+      drain_wait(&ctl->slot_full[n % kSlots], (n / kSlots) & 1);
   } else if (warp == kMmaWarp) {
     // ---------------------------------------------------------- MMA issuer
     constexpr uint32_t idesc_s = idesc_bf16_f32(kHeads, kBlock, false, false);
     constexpr uint32_t idesc_pv = idesc_bf16_f32(kHeads, kChunk, false, true);
-    const uint32_t sQ = smem_addr(smem);
+    const uint32_t sQ8 = smem_addr(smem + kOffQ8);
     const uint32_t sRing = smem_addr(smem + kOffRing);
     bool ok = true;
-    int t = 0;  // chunk step
-    auto take_slot = [&]() -> uint32_t {
-      const int s = t % kSlots;
-      ok = mbar_wait_all(&ctl->slot_full[s], (t / kSlots) & 1, abort);
+    // Partial S(n) = sum over this CTA's chunks of Q_c C_c^T, into S buffer n % 2.
+    auto issue_s = [&](int n) {
+      const int s = n % kSlots, x = n & 1;
+      ok = mbar_wait_all(&ctl->slot_full[s], (n / kSlots) & 1, abort);
       tc_fence_after_sync();
-      return sRing + s * kChunkBytes;
-    };
-    auto release_slot = [&]() {
-      if (elect_one()) umma_commit(&ctl->slot_empty[t % kSlots]);
-      __syncwarp();
-      ++t;
-    };
-    // S(x) = Q C_n^T over the nine key chunks of block n.
-    auto issue_s = [&](int x) {
-      for (int c = 0; ok && c < kChunksK; ++c) {
-        const uint32_t kaddr = take_slot();
-        if (!ok) break;
-        if (elect_one()) {
-          const uint64_t a0 = sdesc_sw128(sQ + c * kHeads * kChunk * 2, 16, 1024);
-          const uint64_t b0 = sdesc_sw128(kaddr, 16, 1024);
+      if (!ok) return;
+      if (elect_one()) {
+        const uint32_t slot = sRing + s * kSlotBytes;
+        const uint32_t d = tmem + kColS + x * kBlock;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          // A = Q chunk from TMEM: 16 components = 8 columns per MMA.
+          const uint64_t b0 = sdesc_sw128(slot + j * kChunkBytes, 16, 1024);
 #pragma unroll
           for (int kk = 0; kk < kChunk / 16; ++kk)
-            umma_ss(tmem + kColS + x * 128, a0 + kk * 2, b0 + kk * 2, idesc_s,
-                    (c > 0 || kk > 0) ? 1u : 0u);
+            umma_ts(d, tmem + kColQ + j * 32 + kk * 8, b0 + kk * 2, idesc_s,
+                    (j > 0 || kk > 0) ? 1u : 0u);
         }
-        __syncwarp();
-        release_slot();
+        if (half == 0) {
+          const uint64_t a0 = sdesc_sw128(sQ8, 16, 1024);
+          const uint64_t b0 = sdesc_sw128(slot + 4 * kChunkBytes, 16, 1024);
+#pragma unroll
+          for (int kk = 0; kk < kChunk / 16; ++kk) umma_ss(d, a0 + kk * 2, b0 + kk * 2, idesc_s, 1u);
+        }
+        umma_commit(&ctl->s_full[x]);
       }
-      if (ok && elect_one()) umma_commit(&ctl->s_full[x]);
       __syncwarp();
     };
-    // O (+)= P(x) C_n[:, value chunks of this CTA]: P is bf16 in the first 64
-    // columns of S buffer x (the TMEM A operand), each value chunk an
-    // MN-major B operand of 128 keys x 64 components.
-    auto issue_pv = [&](int x, bool first_block) {
-      for (int cv = 0; ok && cv < kChunksV; ++cv) {
-        const uint32_t vaddr = take_slot();
-        if (!ok) break;
-        if (elect_one()) {
-          const uint64_t b0 = sdesc_sw128(vaddr, 1024, 1024);
+    // O (+)= P(n) C_n[:, value chunks]: P is bf16 in the first 32 columns of
+    // S buffer n % 2 (the TMEM A operand); each value chunk (positions 0-3 of
+    // the slot) an MN-major B operand of 64 keys x 64 components.
+    auto issue_pv = [&](int n) {
+      const int s = n % kSlots, x = n & 1;
+      if (elect_one()) {
+        const uint32_t slot = sRing + s * kSlotBytes;
+#pragma unroll
+        for (int j = 0; j < kChunksV; ++j) {
+          const uint64_t b0 = sdesc_sw128(slot + j * kChunkBytes, 1024, 1024);
 #pragma unroll
           for (int kk = 0; kk < kBlock / 16; ++kk)
-            umma_ts(tmem + kColO + cv * kChunk, tmem + kColS + x * 128 + kk * 8,
-                    b0 + (uint64_t)(kk * 128), idesc_pv, (!first_block || kk > 0) ? 1u : 0u);
+            umma_ts(tmem + kColO + j * kChunk, tmem + kColS + x * kBlock + kk * 8,
+                    b0 + (uint64_t)(kk * 128), idesc_pv, (n > 0 || kk > 0) ? 1u : 0u);
         }
-        __syncwarp();
-        release_slot();
+        umma_commit(&ctl->pv_done[x]);
+        umma_commit(&ctl->slot_empty[s]);
       }
+      __syncwarp();
     };
     if (nb > 0) {
-      ok = mbar_wait_all(&ctl->q_full, 0, abort);
+      if (half == 0) ok = mbar_wait_all(&ctl->q_full, 0, abort);
+      if (ok) ok = mbar_wait_all(&ctl->qt_full, 0, abort);
+      tc_fence_after_sync();
       if (ok) issue_s(0);
       for (int n = 0; ok && n < nb; ++n) {
         // S(n+1) into the other buffer: its P(n-1) was read by PV(n-1),
         // issued before this.
-        if (n + 1 < nb) issue_s((n + 1) & 1);
+        if (n + 1 < nb) issue_s(n + 1);
         if (!ok) break;
         ok = mbar_wait_all(&ctl->p_full[n & 1], (n >> 1) & 1, abort);
         if (!ok) break;
         tc_fence_after_sync();
-        issue_pv(n & 1, n == 0);
-        if (ok && elect_one()) umma_commit(&ctl->pv_done[n & 1]);
-        __syncwarp();
+        issue_pv(n);
       }
     }
     if (elect_one()) umma_commit(&ctl->mma_drained);
@@ -319,24 +417,78 @@ __global__ void __launch_bounds__(kThreads, 1)
     const float c2 = p.scale_log2;
     float m_run = -INFINITY, l_run = 0.f;
     bool ok = true;
+    if (nb > 0) {
+      // This CTA's four TMEM Q chunks of this head row as bf16 pairs
+      // (component k of chunk position j in the low (k even) or high half of
+      // column kColQ + 32 j + k / 2).  Heads past Hq are zero.
+      const int hq = hg * kHeads + row;
+      const uint4 *qrow = reinterpret_cast<const uint4 *>(p.q + ((int64_t)b * p.Hq + hq) * kDqk +
+                                                          chunk_of(0) * kChunk);
+#pragma unroll 1
+      for (int j = 0; j < 4; ++j) {
+        uint32_t w[32];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const uint4 u = hq < p.Hq ? __ldg(qrow + j * 8 + e) : make_uint4(0u, 0u, 0u, 0u);
+          w[4 * e] = u.x;
+          w[4 * e + 1] = u.y;
+          w[4 * e + 2] = u.z;
+          w[4 * e + 3] = u.w;
+        }
+        tmem_st_32x32b_x32(t_row + kColQ + j * 32, w);
+      }
+      tmem_st_wait();
+      tc_fence_before_sync();
+      mbar_arrive(&ctl->qt_full);
+    }
+    // Exchange slots, laid out [warp][16-byte chunk i of the row][lane]: the
+    // 32 lanes of a warp write (to the partner) and read (locally) 512
+    // contiguous bytes per instruction.
+    const uint32_t exch_own = smem_addr(smem + kOffExch) + warp * 8192 + lane_id() * 16;
+    const uint32_t exch_peer = peer_addr(exch_own, peer);
+    const uint32_t peer_full0 = peer_addr(smem_addr(&ctl->exch_full[0]), peer);
+    const uint32_t peer_full1 = peer_addr(smem_addr(&ctl->exch_full[1]), peer);
+    const uint32_t peer_empty0 = peer_addr(smem_addr(&ctl->exch_empty[0]), peer);
+    const uint32_t peer_empty1 = peer_addr(smem_addr(&ctl->exch_empty[1]), peer);
     for (int n = 0; ok && n < nb; ++n) {
       const int x = n & 1;
       ok = mbar_wait_all(&ctl->s_full[x], (n >> 1) & 1, abort);
       if (!ok) break;
       tc_fence_after_sync();
-      float s[kBlock];
-      {
-        uint32_t raw[4][32];
+      uint32_t raw[kBlock / 32][32];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) tmem_ld_32x32b_x32(t_row + kColS + x * 128 + c * 32, raw[c]);
-        tmem_ld_wait();
+      for (int c = 0; c < kBlock / 32; ++c)
+        tmem_ld_32x32b_x32(t_row + kColS + x * kBlock + c * 32, raw[c]);
+      tmem_ld_wait();
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          reg_fence(raw[c]);
+      for (int c = 0; c < kBlock / 32; ++c) reg_fence(raw[c]);
+      // Send this CTA's partial scores to the partner's slot x once the
+      // partner has read what was there (block n - 2).
+      ok = mbar_wait_cluster(&ctl->exch_empty[x], ((n >> 1) & 1) ^ 1, abort);
+      if (!ok) break;
+      // This CTA's slot x for block n expects the partner's 32 KB.
+      if (threadIdx.x == 0) mbar_arrive_expect_tx(&ctl->exch_full[x], kExchBytes);
 #pragma unroll
-          for (int e = 0; e < 32; ++e) s[c * 32 + e] = __uint_as_float(raw[c][e]) * c2;
-        }
+      for (int i = 0; i < kBlock / 4; ++i) {
+        const uint32_t *w = &raw[i / 8][(i % 8) * 4];
+        st_async_peer_v4(exch_peer + x * kExchBytes + i * 512, w[0], w[1], w[2], w[3],
+                         x ? peer_full1 : peer_full0);
       }
+      // The partner's partial scores of block n, added to this CTA's.
+      ok = mbar_wait_cluster(&ctl->exch_full[x], (n >> 1) & 1, abort);
+      if (!ok) break;
+      float s[kBlock];
+#pragma unroll
+      for (int i = 0; i < kBlock / 4; ++i) {
+        uint32_t a0, a1, a2, a3;
+        ld_shared_v4(exch_own + x * kExchBytes + i * 512, a0, a1, a2, a3);
+        const uint32_t *w = &raw[i / 8][(i % 8) * 4];
+        s[4 * i] = (__uint_as_float(w[0]) + __uint_as_float(a0)) * c2;
+        s[4 * i + 1] = (__uint_as_float(w[1]) + __uint_as_float(a1)) * c2;
+        s[4 * i + 2] = (__uint_as_float(w[2]) + __uint_as_float(a2)) * c2;
+        s[4 * i + 3] = (__uint_as_float(w[3]) + __uint_as_float(a3)) * c2;
+      }
+      mbar_arrive_peer_relaxed(x ? peer_empty1 : peer_empty0);
       const int key0 = (first + n) * kBlock;
       if (key0 + kBlock > L) {
 #pragma unroll
@@ -377,19 +529,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       const float neg_m = m_run == -INFINITY ? 0.f : -m_run;
       float sum0 = 0.f, sum1 = 0.f, sum2 = 0.f, sum3 = 0.f;
-      uint32_t pk[2][32];
+      uint32_t pk[kBlock / 2];
 #pragma unroll
       for (int c = 0; c < kBlock; c += 4) {
         const float p0 = ex2_approx(s[c] + neg_m), p1 = ex2_approx(s[c + 1] + neg_m);
         const float p2 = ex2_approx(s[c + 2] + neg_m), p3 = ex2_approx(s[c + 3] + neg_m);
         fadd2_acc(sum0, sum1, p0, p1);
         fadd2_acc(sum2, sum3, p2, p3);
-        pk[c / 64][(c % 64) / 2] = pack_bf16x2(p0, p1);
-        pk[c / 64][(c % 64) / 2 + 1] = pack_bf16x2(p2, p3);
+        pk[c / 2] = pack_bf16x2(p0, p1);
+        pk[c / 2 + 1] = pack_bf16x2(p2, p3);
       }
       l_run += (sum0 + sum1) + (sum2 + sum3);
-      tmem_st_32x32b_x32(t_row + kColS + x * 128, pk[0]);
-      tmem_st_32x32b_x32(t_row + kColS + x * 128 + 32, pk[1]);
+      tmem_st_32x32b_x32(t_row + kColS + x * kBlock, pk);
       tmem_st_wait();
       tc_fence_before_sync();
       mbar_arrive(&ctl->p_full[x]);
@@ -450,6 +601,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   tc_fence_before_sync();
   __syncthreads();
+  // Neither CTA leaves while the other may still write into its shared
+  // memory or arrive on its barriers.
+  cluster_sync();
   if (warp == kMmaWarp) {
     tc_fence_after_sync();
     tmem_dealloc(tmem, kTmemCols);
@@ -528,7 +682,7 @@ static int sm_count_and_setup() {
   return di.attr == cudaSuccess ? di.sm_count : 0;
 }
 
-// KV splits of whole 128-key blocks: about mla_split_ctas_per_sm (process-wide
+// KV splits of whole 64-key blocks: about mla_split_ctas_per_sm (process-wide
 // tuning) CTAs per SM over B x head groups x 2 value halves.  One CTA fills
 // an SM, so this is the number of waves: more, shorter splits even out
 // unequal sequence lengths, at the cost of a Q load and a merge row each.
@@ -607,6 +761,7 @@ static int mla_decode_impl(const void *q, const void *cache, const int32_t *page
   const int64_t max_keys = (int64_t)max_pages * page_size;
   const int max_blocks = (int)((max_keys + mla::kBlock - 1) / mla::kBlock);
   mla::Params p;
+  p.q = reinterpret_cast<const uint16_t *>(q);
   p.page_table = page_table;
   p.seq_lens = seq_lens;
   p.o = reinterpret_cast<uint16_t *>(o);
@@ -632,14 +787,29 @@ static int mla_decode_impl(const void *q, const void *cache, const int32_t *page
   const cuuint32_t qbox[3] = {(cuuint32_t)mla::kChunk, (cuuint32_t)mla::kHeads, 1};
   const cuuint64_t cdims[2] = {(cuuint64_t)mla::kDqk, (cuuint64_t)num_pages * page_size};
   const cuuint64_t cstr[1] = {(cuuint64_t)mla::kDqk * 2};
-  const cuuint32_t cbox[2] = {(cuuint32_t)mla::kChunk, (cuuint32_t)page_size};
+  const cuuint32_t cbox[2] = {(cuuint32_t)mla::kChunk,
+                             (cuuint32_t)(page_size < mla::kBlock ? page_size : mla::kBlock)};
   if (!mla::encode(&tq, q, 3, qdims, qstr, qbox) || !mla::encode(&tc, cache, 2, cdims, cstr, cbox))
     return MK_ERR_CUDA;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const dim3 grid(2 * B * head_groups, p.n_splits, 1);
   mark_launched(kFamMla);
-  mla::mla_decode_kernel<<<grid, mla::kThreads, mla::kSmemBytes, st>>>(tq, tc, p);
-  if (cudaGetLastError() != cudaSuccess) return MK_ERR_CUDA;
+  {
+    // Clusters of two CTAs along x: the two value halves of one (b, hg, split).
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(mla::kThreads);
+    cfg.dynamicSmemBytes = mla::kSmemBytes;
+    cfg.stream = st;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaLaunchKernelEx(&cfg, mla::mla_decode_kernel, tq, tc, p) != cudaSuccess) return MK_ERR_CUDA;
+  }
   if (p.n_splits > 1) {
     // Scheduled while the decode grid drains; it waits for the partials itself.
     DependentLaunch dl(dim3((B * Hq + 3) / 4), dim3(128), 0, st);
@@ -662,3 +832,4 @@ int mk_attn_mla_decode_paged(const void *q, const void *cache, const int32_t *pa
 }
 
 }  // extern "C"
+
