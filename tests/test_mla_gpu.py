@@ -44,8 +44,9 @@ def check(inp, what):
 @pytest.mark.parametrize("page_size", [16, 32, 64, 128])
 @pytest.mark.parametrize("Hq", [16, 128])
 def test_mla_lengths(page_size, Hq):
-    """Lengths around the 128-key block and page edges, an empty sequence."""
-    lens = [0, 1, 127, 128, 129, page_size + 3, 700, 2049]
+    """Lengths around the 64-key block edges (half a page at page size 128),
+    the page edges and an empty sequence."""
+    lens = [0, 1, 63, 64, 65, 127, 128, 129, 191, 193, page_size + 3, 700, 2049]
     inp = W.make_mla_paged(lens, Hq, page_size, seed=960 + Hq + page_size)
     check(inp, f"ps{page_size} Hq{Hq}")
 
@@ -81,8 +82,8 @@ def test_mla_splits(B):
 
 
 def test_mla_many_sequences():
-    """600 sequences of 0..299 latent rows (page 16, 16 heads): a grid of 1200
-    value-half CTAs per split, empty sequences among them."""
+    """600 sequences of 0..299 latent rows (page 16, 16 heads): a grid of 600
+    two-CTA clusters per split, empty sequences among them."""
     rng = np.random.default_rng(985)
     lens = [int(x) for x in rng.integers(0, 300, size=600)]
     inp = W.make_mla_paged(lens, 16, 16, seed=985)
