@@ -119,3 +119,28 @@ def test_mla_bench_workload():
     lens = [int(x) for x in np.random.default_rng(2001).integers(1024, 8193, size=64)]
     inp = W.make_mla_paged(lens, 128, 64, seed=2002, spare_pages=64)
     check(inp, "bench workload")
+
+
+def test_mla_repeated_calls_are_bitwise_stable():
+    """Back-to-back calls with KV splits (each a grid of two-CTA clusters that
+    exchange partial scores through distributed shared memory) give the same
+    bits every time and leave the status word clean: a race in the exchange
+    or in the split merge would show up as a differing call."""
+    dev = torch.device("cuda")
+    inp = W.make_mla_paged([4000, 1, 0, 2500, 63, 65, 129], 128, 16, seed=993)
+    args = [t.to(dev).contiguous() for t in (inp.q, inp.cache, inp.page_table, inp.seq_lens)]
+    B, Hq, _ = inp.q.shape
+    need = binding.mk_attn_mla_decode_workspace_bytes(B, Hq, inp.cache.shape[1], inp.page_table.shape[1])
+    assert need > 0, "the case must use several KV splits"
+    ws = torch.empty(need // 4 + 4, dtype=torch.float32, device=dev)
+    o0 = torch.empty((B, Hq, binding.MLA_DV), dtype=torch.bfloat16, device=dev)
+    l0 = torch.empty((B, Hq), dtype=torch.float32, device=dev)
+    binding.mla_decode_paged(*args, scale=inp.scale, out=o0, lse=l0, workspace=ws)
+    o = torch.empty_like(o0)
+    l = torch.empty_like(l0)
+    for _ in range(40):
+        o.fill_(float("nan"))
+        binding.mla_decode_paged(*args, scale=inp.scale, out=o, lse=l, workspace=ws)
+        torch.cuda.synchronize()
+        assert torch.equal(o.view(torch.int16), o0.view(torch.int16)) and torch.equal(l, l0)
+    assert binding.mk_attn_check_status(torch.cuda.current_stream().cuda_stream) == binding.MK_OK
